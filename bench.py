@@ -1,0 +1,393 @@
+"""Benchmark of the memory-planning path on GB300: one JSON line on stdout.
+
+A step is one pass of the whole path -- live-bytes profile, greedy_by_size
+plan (with its peak) and pairwise validation -- over the batched workload of
+4096 random traces (512 tensors over T = 1024 steps each, seeds 0..4095; rank
+r of a multi-GPU run takes seeds r*4096 .. r*4096+4095: weak scaling, no
+collective on the data path).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--policy first|best]
+    python bench.py --impl reference ...   # the CPU oracle as the reference arm
+
+Timing: W untimed warm-up steps; then K steps, each preceded by an L2 flush
+(256 MiB device write, outside the timed events) and timed with CUDA events
+on the launching stream; barrier + synchronize on both sides of the K-step
+region; the max over ranks is reported.  Per-kernel events give the dominant
+kernel's achieved bandwidth for the roofline object.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "greedy-by-size tensors planned/s and validated pairs/s on 1 GB300 (% HBM roofline)"
+UNIT = "tensors/s"
+WORKLOAD = dict(n_traces=4096, n=512, T=1024, p=0.5, lo_e=6, hi_e=20)
+WORKLOAD_NAME = "batched-random-4096x512x1024-seeds0-4095"
+FALLBACK_HBM_GBS = 6800.0
+L2_FLUSH_BYTES = 256 << 20
+
+# Algorithmic bytes per unit (what each kernel must move at minimum).
+# profile : read alloc/free/size 16 B per tensor and trace_ptr/steps/profile_ptr 20 B
+#           per trace; write 8 B per step, peak_lb 8 B and status 4 B per trace.
+# plan    : read 16 B per tensor and 12 B per trace; write offsets 8 B per tensor,
+#           plan_peak 8 B and status 4 B per trace.
+# validate: read alloc/free/size/offset 24 B per tensor and 12 B per trace; write
+#           verdict 4 B, conflict 8 B and status 4 B per trace.
+KERNELS = ("live_profile", "plan_greedy_by_size", "validate_plan")
+
+
+def algorithmic_bytes(kernel: str, n_tensors: int, n_traces: int, n_steps: int) -> int:
+    if kernel == "live_profile":
+        return 16 * n_tensors + 8 * n_steps + (20 + 12) * n_traces
+    if kernel == "plan_greedy_by_size":
+        return 24 * n_tensors + (12 + 12) * n_traces
+    if kernel == "validate_plan":
+        return 24 * n_tensors + (12 + 16) * n_traces
+    raise KeyError(kernel)
+
+
+# ----------------------------------------------------------------- distributed helpers
+
+def dist_env():
+    """(rank, world, local_rank) from the torchrun environment (1 process if absent)."""
+    return int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)), int(os.environ.get("LOCAL_RANK", 0))
+
+
+def shard_seed0(rank: int, n_traces: int = WORKLOAD["n_traces"]) -> int:
+    """First seed of this rank's batch (weak scaling: every rank plans its own batch)."""
+    return rank * n_traces
+
+
+def max_over_ranks(value: float, dist=None) -> float:
+    if dist is None or not dist.is_initialized() or dist.get_world_size() == 1:
+        return value
+    import torch
+
+    backend = dist.get_backend()
+    dev = torch.device("cuda", torch.cuda.current_device()) if backend == "nccl" else torch.device("cpu")
+    t = torch.tensor([value], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(value: float, dist=None) -> float:
+    if dist is None or not dist.is_initialized() or dist.get_world_size() == 1:
+        return value
+    import torch
+
+    backend = dist.get_backend()
+    dev = torch.device("cuda", torch.cuda.current_device()) if backend == "nccl" else torch.device("cpu")
+    t = torch.tensor([value], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+# ----------------------------------------------------------------- measurement helpers
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_digest() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2203_00448_gb300", "csrc")
+    for fn in sorted(os.listdir(csrc)):
+        if fn.endswith((".cu", ".cuh", ".h")):
+            h.update(open(os.path.join(csrc, fn), "rb").read())
+    return h.hexdigest()
+
+
+def ncu_traffic(kernel: str, n_tensors: int):
+    """DRAM bytes per launch from the committed ncu capture, scaled to this
+    launch's tensor count; None if absent or if the kernels changed since."""
+    path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+    except (OSError, ValueError):
+        return None
+    if d.get("source_sha256") != kernel_source_digest():
+        return None
+    k = d.get("kernels", {}).get(kernel)
+    if not k:
+        return None
+    return k["dram_bytes"] * n_tensors / k["n_tensors"]
+
+
+def gpu_id(dev) -> str:
+    """nvidia-smi --id value for a torch device (its UUID, else its index)."""
+    import torch
+
+    uuid = getattr(torch.cuda.get_device_properties(dev), "uuid", None)
+    if uuid is not None:
+        u = str(uuid)
+        return u if u.startswith("GPU-") else "GPU-" + u
+    return str(dev.index or 0)
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling during the timed region."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.out = ""
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                self.out, _ = self.proc.communicate()
+
+    def summary(self):
+        rows = [r.split(",") for r in (self.out or "").strip().splitlines() if r.count(",") >= 8]
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        sm = [float(r[1]) for r in rows if r[1].strip().replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].strip().replace(".", "").isdigit()]
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        reasons = sorted({names[k] for r in rows for k in range(4) if r[5 + k].strip() == "Active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+# ----------------------------------------------------------------- CPU oracle baseline
+
+def oracle_baseline(ts, n_sample_traces: int):
+    """The oracle as it stands, single-threaded on the host: profile + plan +
+    validate over the first `n_sample_traces` traces of the workload."""
+    import oracle
+
+    sub = ts.select(range(min(n_sample_traces, ts.n_traces)))
+    t0 = time.perf_counter()
+    oracle.live_profile(sub)
+    off, _, _ = oracle.plan_greedy_by_size(sub, oracle.FIT_FIRST)
+    oracle.validate_plan(sub, off)
+    dt = time.perf_counter() - t0
+    return sub.n_tensors / dt, dt, sub
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    import tracegen
+
+    w = WORKLOAD
+    ts = tracegen.random_batch(0, w["n_traces"], w["n"], w["T"], w["p"], w["lo_e"], w["hi_e"], name=WORKLOAD_NAME)
+    sample = 512
+    for _ in range(args.warmup):
+        oracle_baseline(ts, sample)
+    times, n = [], 0
+    for _ in range(args.steps):
+        _, dt, sub = oracle_baseline(ts, sample)
+        times.append(dt)
+        n = sub.n_tensors
+    total = sum(times)
+    value = n * args.steps / total
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64",
+        "data": "synthetic", "config": {"workload": WORKLOAD_NAME, "policy": "first", "n_traces_per_step": sample},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": f"first {sample} of the 4096 traces per step (profile + plan + validate)"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    return 0
+
+
+# ----------------------------------------------------------------- GPU arm
+
+def run_gpu(args):
+    import torch
+
+    rank, world, local = dist_env()
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    import paper_2203_00448_gb300 as mp
+    import tracegen
+    from paper_2203_00448_gb300 import build
+
+    build.build()
+    w = WORKLOAD
+    ts = tracegen.random_batch(shard_seed0(rank), w["n_traces"], w["n"], w["T"], w["p"], w["lo_e"], w["hi_e"],
+                               name=WORKLOAD_NAME)
+    dev = torch.device("cuda", torch.cuda.current_device())
+    db = mp.DeviceBatch.from_host(ts, dev)
+    buf = mp.PathBuffers(db)
+    stream = torch.cuda.current_stream()
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+
+    def step(ev=None):
+        if ev is not None:
+            ev[0].record(stream)
+        mp.live_profile(db, buf.profile, buf.peak_lb, buf.status[0], stream=stream)
+        if ev is not None:
+            ev[1].record(stream)
+        mp.plan_greedy_by_size(db, args.policy, buf.offsets, buf.plan_peak, buf.status[1], workspace=buf.plan_ws,
+                               stream=stream)
+        if ev is not None:
+            ev[2].record(stream)
+        mp.validate_plan(db, buf.offsets, buf.verdict, buf.conflict, buf.status[2], workspace=buf.validate_ws,
+                         stream=stream)
+        if ev is not None:
+            ev[3].record(stream)
+
+    for _ in range(args.warmup):
+        flush.zero_()
+        step()
+    torch.cuda.synchronize()
+    st = buf.status.cpu()
+    if not bool((st == 0).all()) or not bool((buf.verdict == 1).all()):
+        print(json.dumps({"error": "path reported a failed trace or an invalid plan", "rank": rank}))
+        return 1
+
+    events = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    sampler = ClockSampler(gpu_id(dev))
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with sampler:
+        t0 = time.perf_counter()
+        for k in range(args.steps):
+            flush.zero_()
+            step(events[k])
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - t0
+    if dist is not None:
+        dist.barrier()
+    per_kernel = [0.0, 0.0, 0.0]
+    step_ms = 0.0
+    for ev in events:
+        for j in range(3):
+            per_kernel[j] += ev[j].elapsed_time(ev[j + 1])
+        step_ms += ev[0].elapsed_time(ev[3])
+    step_ms /= args.steps
+    per_kernel = [x / args.steps for x in per_kernel]
+    step_ms_max = max_over_ranks(step_ms, dist)
+    wall_max = max_over_ranks(wall, dist)
+    total_tensors = sum_over_ranks(float(ts.n_tensors), dist)
+    total_pairs = sum_over_ranks(float(ts.pairs()), dist)
+
+    # End to end through the host-buffer API: pinned H2D of the inputs, the
+    # path, and D2H of every result, each step.
+    e2e = None
+    if not args.no_e2e:
+        hp = mp.HostPath(ts, dev, args.policy, stream=stream)
+        hp.stage(ts)
+        for _ in range(max(1, args.warmup)):
+            hp.run()
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize()
+        e2e_steps = max(3, args.steps // 2)
+        t0 = time.perf_counter()
+        for _ in range(e2e_steps):
+            hp.run()
+        e2e_s = max_over_ranks((time.perf_counter() - t0) / e2e_steps, dist)
+        e2e = {"value": total_tensors / e2e_s, "unit": UNIT, "h2d_bytes_per_step": hp.h2d_bytes,
+               "d2h_bytes_per_step": hp.d2h_bytes, "ms_per_step": 1e3 * e2e_s}
+
+    if rank != 0:
+        if dist is not None:
+            dist.destroy_process_group()
+        return 0
+    peak, peak_kind = measured_peaks()
+    n_steps = ts.n_steps
+    kern = {}
+    for j, name in enumerate(KERNELS):
+        nbytes = algorithmic_bytes(name, ts.n_tensors, ts.n_traces, n_steps)
+        gbs = nbytes / (per_kernel[j] * 1e-3) / 1e9
+        kern[name] = {"ms": per_kernel[j], "algorithmic_bytes": nbytes, "achieved_gbs": gbs,
+                      "frac": gbs / peak, "share": per_kernel[j] / sum(per_kernel)}
+    dom = max(KERNELS, key=lambda k: kern[k]["ms"])
+    traffic = ncu_traffic(dom, ts.n_tensors)
+    roof = {"bound": "hbm", "kernel": dom, "achieved": kern[dom]["achieved_gbs"], "peak": peak, "unit": "GB/s",
+            "frac": kern[dom]["frac"], "peak_source": f"{peak_kind} ({'MEASURED_PEAKS.json hbm_gbs' if peak_kind == 'measured' else 'profiling-recipe fallback'})",
+            "traffic": traffic}
+    ob_value, ob_dt, ob_sub = oracle_baseline(ts, args.oracle_traces)
+    clocks = sampler.summary()
+    line = {
+        "metric": METRIC, "value": total_tensors / (step_ms_max * 1e-3), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms_max, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+        "config": {"workload": WORKLOAD_NAME, "n_traces": ts.n_traces * world, "tensors_per_trace": w["n"],
+                   "steps_per_trace": w["T"], "policy": args.policy,
+                   "l2": "flushed before every timed step (256 MiB device write outside the timed events)",
+                   "parallelism": f"dp{world} (traces sharded by rank, no collective)"},
+        "validated_pairs_per_s": total_pairs / (step_ms_max * 1e-3),
+        "wall_ms_per_step_incl_flush": 1e3 * wall_max / args.steps,
+        "gpu_launches": 3 * args.steps,
+        "kernels": kern,
+        "roofline": roof,
+        "cpu_baseline": {"value": ob_value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": f"first {ob_sub.n_traces} of {ts.n_traces} traces, profile + plan + validate, "
+                                   f"{ob_dt:.2f} s single-threaded"},
+        "e2e": e2e,
+        "clocks": clocks,
+    }
+    print(json.dumps(line))
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--policy", choices=("first", "best"), default="first")
+    ap.add_argument("--oracle-traces", type=int, default=4096,
+                    help="traces of the workload the CPU-baseline leg runs through the oracle")
+    ap.add_argument("--no-e2e", action="store_true")
+    args = ap.parse_args(argv)
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_gpu(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

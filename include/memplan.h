@@ -1,0 +1,160 @@
+/*
+ * memplan.h -- C ABI of the GB300 memory-planning library (libmemplan.so).
+ *
+ * The library builds and checks static memory plans for batches of
+ * allocation traces, the static-analysis half of MemoMalloc ("Memory Planning
+ * for Deep Neural Networks", arXiv 2203.00448).  A trace lists the
+ * intermediate tensors of one forward pass; tensor i has a lifetime
+ * [alloc_step_i, free_step_i) over op steps (half-open) and a size in bytes.
+ * A plan gives every tensor an offset into one slab (Sec. 3.3,
+ * prim::AllocateSlab[total_size] / prim::AllocateTensor[size, offset]).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - All array pointers inside mp_batch and all output pointers are DEVICE
+ *   pointers (cudaMalloc'd or managed), owned by the caller; the library never
+ *   frees or retains them.  The mp_batch struct itself is read on the host
+ *   during the call and may be discarded afterwards.
+ * - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *   Every call only enqueues work on that stream and returns without
+ *   synchronising; outputs are valid once the stream reaches that point.
+ * - The return value reports host-side problems only: MP_EINVAL for a NULL
+ *   or misaligned pointer, a negative count or a too-small workspace;
+ *   MP_ECUDA when a launch fails.  On any non-OK return nothing was enqueued.
+ * - Per-trace data errors are written to trace_status[b] on the device:
+ *     MP_EINVAL    bad CSR range (trace_ptr not non-decreasing, beyond
+ *                  n_tensors, or more than max_tensors tensors), T_b < 0 or
+ *                  T_b > max_steps, a tensor with alloc < 0, free <= alloc,
+ *                  free > T_b or size <= 0, or (where offsets are inputs)
+ *                  offset < 0;
+ *     MP_EOVERFLOW the sizes of the trace sum past INT64_MAX, or (where
+ *                  offsets are inputs) some offset + size does;
+ *   EINVAL takes precedence.  Outputs of a failed trace are unspecified but
+ *   nothing outside that trace's own output range is written.
+ * - Tensor ids are local indices within their trace.  A trace with no
+ *   tensors is valid; its profile is all zero and both peaks are 0.
+ * - All arithmetic is integer (int64 bytes/offsets, int32 steps/ids), so
+ *   results are bit-identical to the plain definitions, whatever the launch
+ *   configuration.
+ */
+#ifndef MEMPLAN_H
+#define MEMPLAN_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum mp_status {
+    MP_OK = 0,
+    MP_EINVAL = 1,
+    MP_EOVERFLOW = 2,
+    MP_ECUDA = 3,
+    MP_ETIMEOUT = 4, /* reserved for waits that give up; no entry point waits today */
+    MP_ENOMEM = 5,   /* workspace smaller than the matching *_workspace_bytes */
+    MP_EINTERNAL = 6 /* per-trace only: a kernel found an inconsistency in its own
+                        state (a library defect); that trace's outputs are unspecified */
+} mp_status;
+
+/* Fit criterion of greedy_by_size.  Sec. 2.3 describes a best-fit criterion;
+ * first fit is the lowest feasible offset.  Both are exact. */
+typedef enum mp_fit_policy { MP_FIT_FIRST = 0, MP_FIT_BEST = 1 } mp_fit_policy;
+
+/* A batch of B traces as a structure of arrays with CSR offsets.
+ * Host scalars (read on the host, used to size launches and workspace):
+ *   n_traces     B >= 0
+ *   max_tensors  upper bound on N_b = trace_ptr[b+1] - trace_ptr[b]
+ *   max_steps    upper bound on T_b
+ *   n_tensors    length of alloc_step / free_step / size_bytes (= trace_ptr[B])
+ *   n_steps      length of the profile output (= profile_ptr[B])
+ * A trace breaking a declared bound is rejected with MP_EINVAL in
+ * trace_status; it never causes an access outside the arrays.
+ * Device arrays:
+ *   trace_ptr    int64[B+1]  tensors of trace b: [trace_ptr[b], trace_ptr[b+1])
+ *   steps        int32[B]    T_b, number of op steps of trace b
+ *   profile_ptr  int64[B+1]  profile of trace b: [profile_ptr[b], +T_b);
+ *                            only mp_live_profile reads it (may be NULL elsewhere)
+ *   alloc_step   int32[n_tensors]  first live step
+ *   free_step    int32[n_tensors]  first step no longer live (exclusive)
+ *   size_bytes   int64[n_tensors]  size, >= 1
+ * int64 arrays must be 8-byte aligned, int32 arrays 4-byte aligned. */
+typedef struct mp_batch {
+    int32_t n_traces;
+    int32_t max_tensors;
+    int32_t max_steps;
+    int32_t reserved0; /* must be 0 */
+    int64_t n_tensors;
+    int64_t n_steps;
+    const int64_t *trace_ptr;
+    const int32_t *steps;
+    const int64_t *profile_ptr;
+    const int32_t *alloc_step;
+    const int32_t *free_step;
+    const int64_t *size_bytes;
+} mp_batch;
+
+/* Live-bytes profile and its peak (stage 1).
+ * profile[profile_ptr[b] + t] = sum of size_i over tensors with
+ *   alloc_i <= t < free_i, for 0 <= t < T_b                      int64[n_steps]
+ * peak_lb[b] = max_t profile (0 when T_b = 0): every feasible total_mem of
+ *   Eq. 2.1 is at least this, because the tensors live at one step must all
+ *   fit side by side (Sec. 1 and Sec. 2.3).                        int64[B]
+ * trace_status[b]                                                   int32[B]
+ * Needs no workspace (the profile output doubles as the difference array). */
+mp_status mp_live_profile(const mp_batch *batch, int64_t *profile, int64_t *peak_lb,
+                          int32_t *trace_status, void *stream);
+
+/* Bytes of device workspace mp_plan_greedy_by_size needs for this batch
+ * (depends on the host scalars only).  0 means none. */
+size_t mp_plan_workspace_bytes(const mp_batch *batch);
+
+/* greedy_by_size offset assignment (stage 2; Sec. 2.3, default strategy of
+ * Sec. 3.2).  Tensors are taken in priority order -- size descending, then
+ * alloc_step ascending, then id ascending -- and each is given, among the
+ * already placed tensors whose lifetimes overlap its own, the first gap
+ * (MP_FIT_FIRST: the lowest offset where it fits) or the smallest gap that
+ * fits, lowest on ties (MP_FIT_BEST), gaps being measured against the running
+ * maximum end in address order; if no gap fits it goes above them all.
+ * offsets[trace_ptr[b] + i]   int64[n_tensors]
+ * plan_peak[b] = max_i offset_i + size_i, the plan's total_mem   int64[B]
+ * trace_status[b]                                               int32[B]
+ * max_tensors must be below 2^28 (MP_EINVAL otherwise).
+ * workspace: device memory of at least mp_plan_workspace_bytes(batch) bytes,
+ * 256-byte aligned, owned by the caller, not used concurrently by another
+ * call.  Its contents need not be initialised. */
+mp_status mp_plan_greedy_by_size(const mp_batch *batch, mp_fit_policy policy, int64_t *offsets,
+                                 int64_t *plan_peak, int32_t *trace_status, void *workspace,
+                                 size_t workspace_bytes, void *stream);
+
+/* Bytes of device workspace mp_validate_plan needs for this batch. */
+size_t mp_validate_workspace_bytes(const mp_batch *batch);
+
+/* Plan validation (stage 3; pairwise constraints of Eq. 2.1).
+ * verdict[b] = 1 iff for all i < j with overlapping lifetimes the address
+ *   ranges [offset, offset + size) are disjoint (touching is allowed), else 0.
+ * conflict[2b], conflict[2b+1] = the violating pair (i, j), i < j, with the
+ *   smallest i and then the smallest j, or (-1, -1); may be NULL.
+ * offsets: int64[n_tensors] device array, one per tensor.
+ * workspace as for mp_plan_greedy_by_size, sized by
+ * mp_validate_workspace_bytes. */
+mp_status mp_validate_plan(const mp_batch *batch, const int64_t *offsets, int32_t *verdict,
+                           int32_t *conflict, int32_t *trace_status, void *workspace,
+                           size_t workspace_bytes, void *stream);
+
+/* Peak of a given plan: plan_peak[b] = max_i offset_i + size_i (0 for an
+ * empty trace), Eq. 2.1's total_mem.  Needs no workspace. */
+mp_status mp_peak(const mp_batch *batch, const int64_t *offsets, int64_t *plan_peak,
+                  int32_t *trace_status, void *stream);
+
+/* Static, NUL-terminated name of a status code. */
+const char *mp_status_string(mp_status status);
+
+/* ABI version of this header (incremented on incompatible changes). */
+int32_t mp_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MEMPLAN_H */

@@ -1,0 +1,287 @@
+"""Python binding of the memory-planning C ABI (argument marshalling only).
+
+Device memory and streams come from PyTorch; every step of the path runs in
+libmemplan.so's CUDA kernels.  Function names follow the C ABI:
+
+    live_profile(batch)                  -> profile, peak_lb, status     (stage 1)
+    plan_greedy_by_size(batch, policy)   -> offsets, plan_peak, status   (stage 2)
+    validate_plan(batch, offsets)        -> verdict, conflict, status    (stage 3)
+    peak(batch, offsets)                 -> plan_peak, status
+
+All calls are asynchronous on the current (or given) CUDA stream.
+"""
+from __future__ import annotations
+
+import ctypes
+from dataclasses import dataclass
+
+import torch
+
+from . import _lib
+from ._lib import FIT_BEST, FIT_FIRST, MemplanError, MpBatch
+
+_POLICIES = {"first": FIT_FIRST, "best": FIT_BEST, FIT_FIRST: FIT_FIRST, FIT_BEST: FIT_BEST}
+
+
+def _policy(p) -> int:
+    try:
+        return _POLICIES[p]
+    except KeyError:
+        raise ValueError(f"unknown fit policy {p!r}; use 'first' or 'best'") from None
+
+
+def _stream_ptr(stream) -> int:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return int(stream.cuda_stream)
+
+
+def _ptr(t):
+    return None if t is None or t.numel() == 0 else t.data_ptr()
+
+
+@dataclass
+class DeviceBatch:
+    """A batch of traces resident on one CUDA device (structure of arrays + CSR).
+
+    The host scalars (n_traces, max_tensors, max_steps, n_tensors, n_steps)
+    size launches and workspace; the kernels re-check every trace against
+    them.
+    """
+
+    trace_ptr: torch.Tensor
+    steps: torch.Tensor
+    profile_ptr: torch.Tensor
+    alloc_step: torch.Tensor
+    free_step: torch.Tensor
+    size_bytes: torch.Tensor
+    n_traces: int
+    max_tensors: int
+    max_steps: int
+    n_tensors: int
+    n_steps: int
+
+    @classmethod
+    def from_host(cls, ts, device="cuda", non_blocking: bool = False) -> "DeviceBatch":
+        """Copies a host batch (numpy arrays, e.g. tracegen.TraceSet) to `device`."""
+        def dev(a, dt):
+            t = torch.as_tensor(a).to(dt)
+            return t.to(device, non_blocking=non_blocking)
+
+        return cls(
+            trace_ptr=dev(ts.trace_ptr, torch.int64),
+            steps=dev(ts.steps, torch.int32),
+            profile_ptr=dev(ts.profile_ptr, torch.int64),
+            alloc_step=dev(ts.alloc_step, torch.int32),
+            free_step=dev(ts.free_step, torch.int32),
+            size_bytes=dev(ts.size_bytes, torch.int64),
+            n_traces=int(ts.n_traces),
+            max_tensors=int(ts.max_tensors),
+            max_steps=int(ts.max_steps),
+            n_tensors=int(ts.n_tensors),
+            n_steps=int(ts.n_steps),
+        )
+
+    @property
+    def device(self) -> torch.device:
+        return self.alloc_step.device
+
+    def struct(self) -> MpBatch:
+        return MpBatch(self.n_traces, self.max_tensors, self.max_steps, 0, self.n_tensors, self.n_steps,
+                       _ptr(self.trace_ptr), _ptr(self.steps), _ptr(self.profile_ptr), _ptr(self.alloc_step),
+                       _ptr(self.free_step), _ptr(self.size_bytes))
+
+
+class Workspace:
+    """Caller-owned scratch for the calls that need it; grows on demand, never shrinks."""
+
+    def __init__(self, device="cuda"):
+        self.device = torch.device(device)
+        self.buf = None
+
+    def get(self, nbytes: int):
+        if nbytes == 0:
+            return None, 0
+        if self.buf is None or self.buf.numel() < nbytes:
+            # 256-byte alignment: the caching allocator returns 512-byte aligned blocks
+            self.buf = torch.empty(nbytes, dtype=torch.uint8, device=self.device)
+        return self.buf.data_ptr(), self.buf.numel()
+
+
+_default_ws = {}
+
+
+def _workspace(ws, device):
+    if ws is not None:
+        return ws
+    key = torch.device(device)
+    if key not in _default_ws:
+        _default_ws[key] = Workspace(key)
+    return _default_ws[key]
+
+
+def _check(fn, st):
+    if st != _lib.OK:
+        raise MemplanError(fn, st)
+
+
+def _empty(n, dtype, device):
+    return torch.empty(max(int(n), 0), dtype=dtype, device=device)
+
+
+def plan_workspace_bytes(batch: DeviceBatch) -> int:
+    s = batch.struct()
+    return int(_lib.load().mp_plan_workspace_bytes(ctypes.byref(s)))
+
+
+def validate_workspace_bytes(batch: DeviceBatch) -> int:
+    s = batch.struct()
+    return int(_lib.load().mp_validate_workspace_bytes(ctypes.byref(s)))
+
+
+def live_profile(batch: DeviceBatch, profile=None, peak_lb=None, status=None, stream=None):
+    """Stage 1: live bytes per step (int64[n_steps]) and its max per trace."""
+    lib, dev = _lib.load(), batch.device
+    profile = _empty(batch.n_steps, torch.int64, dev) if profile is None else profile
+    peak_lb = _empty(batch.n_traces, torch.int64, dev) if peak_lb is None else peak_lb
+    status = _empty(batch.n_traces, torch.int32, dev) if status is None else status
+    s = batch.struct()
+    _check("mp_live_profile", lib.mp_live_profile(ctypes.byref(s), _ptr(profile), _ptr(peak_lb), _ptr(status),
+                                                  _stream_ptr(stream)))
+    return profile, peak_lb, status
+
+
+def plan_greedy_by_size(batch: DeviceBatch, policy="first", offsets=None, plan_peak=None, status=None,
+                        workspace: Workspace | None = None, stream=None):
+    """Stage 2: greedy_by_size offsets (int64[n_tensors]) and the plan peak per trace."""
+    lib, dev = _lib.load(), batch.device
+    offsets = _empty(batch.n_tensors, torch.int64, dev) if offsets is None else offsets
+    plan_peak = _empty(batch.n_traces, torch.int64, dev) if plan_peak is None else plan_peak
+    status = _empty(batch.n_traces, torch.int32, dev) if status is None else status
+    s = batch.struct()
+    need = int(lib.mp_plan_workspace_bytes(ctypes.byref(s)))
+    wptr, wbytes = _workspace(workspace, dev).get(need)
+    _check("mp_plan_greedy_by_size",
+           lib.mp_plan_greedy_by_size(ctypes.byref(s), _policy(policy), _ptr(offsets), _ptr(plan_peak),
+                                      _ptr(status), wptr, wbytes, _stream_ptr(stream)))
+    return offsets, plan_peak, status
+
+
+def validate_plan(batch: DeviceBatch, offsets: torch.Tensor, verdict=None, conflict=None, status=None,
+                  workspace: Workspace | None = None, stream=None, want_conflict: bool = True):
+    """Stage 3: per-trace verdict (1 valid) and first conflicting pair (int32[B, 2])."""
+    lib, dev = _lib.load(), batch.device
+    verdict = _empty(batch.n_traces, torch.int32, dev) if verdict is None else verdict
+    if conflict is None and want_conflict:
+        conflict = _empty(2 * batch.n_traces, torch.int32, dev)
+    status = _empty(batch.n_traces, torch.int32, dev) if status is None else status
+    s = batch.struct()
+    need = int(lib.mp_validate_workspace_bytes(ctypes.byref(s)))
+    wptr, wbytes = _workspace(workspace, dev).get(need)
+    _check("mp_validate_plan",
+           lib.mp_validate_plan(ctypes.byref(s), _ptr(offsets), _ptr(verdict), _ptr(conflict), _ptr(status),
+                                wptr, wbytes, _stream_ptr(stream)))
+    return verdict, (conflict.view(-1, 2) if conflict is not None else None), status
+
+
+def peak(batch: DeviceBatch, offsets: torch.Tensor, plan_peak=None, status=None, stream=None):
+    """total_mem of a given plan per trace: max(offset + size)."""
+    lib, dev = _lib.load(), batch.device
+    plan_peak = _empty(batch.n_traces, torch.int64, dev) if plan_peak is None else plan_peak
+    status = _empty(batch.n_traces, torch.int32, dev) if status is None else status
+    s = batch.struct()
+    _check("mp_peak", lib.mp_peak(ctypes.byref(s), _ptr(offsets), _ptr(plan_peak), _ptr(status),
+                                  _stream_ptr(stream)))
+    return plan_peak, status
+
+
+@dataclass
+class PathResult:
+    profile: torch.Tensor
+    peak_lb: torch.Tensor
+    offsets: torch.Tensor
+    plan_peak: torch.Tensor
+    verdict: torch.Tensor
+    conflict: torch.Tensor
+    status: torch.Tensor  # int32[3, B]: profile, plan, validate
+
+
+class PathBuffers:
+    """Preallocated outputs for repeated runs of the whole path on one batch."""
+
+    def __init__(self, batch: DeviceBatch):
+        dev = batch.device
+        B = batch.n_traces
+        self.profile = _empty(batch.n_steps, torch.int64, dev)
+        self.peak_lb = _empty(B, torch.int64, dev)
+        self.offsets = _empty(batch.n_tensors, torch.int64, dev)
+        self.plan_peak = _empty(B, torch.int64, dev)
+        self.verdict = _empty(B, torch.int32, dev)
+        self.conflict = _empty(2 * B, torch.int32, dev)
+        self.status = torch.empty((3, B), dtype=torch.int32, device=dev)
+        self.plan_ws = Workspace(dev)
+        self.validate_ws = Workspace(dev)
+        self.plan_ws.get(plan_workspace_bytes(batch))
+        self.validate_ws.get(validate_workspace_bytes(batch))
+
+
+def run_path(batch: DeviceBatch, policy="first", buffers: PathBuffers | None = None, stream=None) -> PathResult:
+    """One pass of the whole path: profile, greedy_by_size plan (with its peak), validation."""
+    buf = buffers or PathBuffers(batch)
+    live_profile(batch, buf.profile, buf.peak_lb, buf.status[0], stream=stream)
+    plan_greedy_by_size(batch, policy, buf.offsets, buf.plan_peak, buf.status[1], workspace=buf.plan_ws,
+                        stream=stream)
+    validate_plan(batch, buf.offsets, buf.verdict, buf.conflict, buf.status[2], workspace=buf.validate_ws,
+                  stream=stream)
+    return PathResult(buf.profile, buf.peak_lb, buf.offsets, buf.plan_peak, buf.verdict,
+                      buf.conflict.view(-1, 2), buf.status)
+
+
+class HostPath:
+    """End-to-end use from host memory: copies a batch from pinned host buffers
+    to the device, runs the whole path, and copies every result back.
+
+    ``run(ts)`` takes a host batch (numpy arrays, e.g. tracegen.TraceSet) with
+    the same shape as the one the object was built for and returns host
+    numpy views of profile, peak_lb, offsets, plan_peak, verdict, conflict,
+    status.  All copies are stream-ordered on the given stream.
+    """
+
+    _IN = ("trace_ptr", "steps", "profile_ptr", "alloc_step", "free_step", "size_bytes")
+
+    def __init__(self, ts, device="cuda", policy="first", stream=None):
+        self.policy = policy
+        self.stream = stream
+        self.dev_batch = DeviceBatch.from_host(ts, device)
+        self.buffers = PathBuffers(self.dev_batch)
+        self.host_in = {k: torch.empty(tuple(getattr(self.dev_batch, k).shape), dtype=getattr(self.dev_batch, k).dtype,
+                                       pin_memory=True) for k in self._IN}
+        self._outs = ("profile", "peak_lb", "offsets", "plan_peak", "verdict", "conflict", "status")
+        self.host_out = {k: torch.empty(tuple(getattr(self.buffers, k).shape), dtype=getattr(self.buffers, k).dtype,
+                                        pin_memory=True) for k in self._outs}
+
+    @property
+    def h2d_bytes(self) -> int:
+        return sum(t.numel() * t.element_size() for t in self.host_in.values())
+
+    @property
+    def d2h_bytes(self) -> int:
+        return sum(t.numel() * t.element_size() for t in self.host_out.values())
+
+    def stage(self, ts):
+        """Places a host batch into the pinned input buffers (host-side memcpy)."""
+        for k in self._IN:
+            self.host_in[k].numpy()[...] = getattr(ts, k)
+
+    def run(self, ts=None):
+        if ts is not None:
+            self.stage(ts)
+        s = self.stream or torch.cuda.current_stream()
+        with torch.cuda.stream(s):
+            for k in self._IN:
+                getattr(self.dev_batch, k).copy_(self.host_in[k], non_blocking=True)
+            run_path(self.dev_batch, self.policy, self.buffers, stream=s)
+            for k in self._outs:
+                self.host_out[k].copy_(getattr(self.buffers, k), non_blocking=True)
+        s.synchronize()
+        return {k: v.numpy() for k, v in self.host_out.items()}

@@ -1,0 +1,50 @@
+// launch.h -- internal launch interface between the C ABI (abi.cu) and the
+// kernel translation units.  Not part of the public header.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "memplan.h"
+
+namespace mp {
+
+constexpr int kProfileThreads = 256;
+constexpr int kValidateThreads = 256;
+constexpr int kPeakThreads = 256;
+constexpr int kPlanThreadsSmem = 256;    // one CTA per trace, data in shared memory
+constexpr int kPlanThreadsGlobal = 1024; // one CTA per trace, data in the workspace
+
+// Largest dynamic shared memory a kernel of this library requests per CTA
+// (sm_103a allows 227 KB); above it a kernel keeps its data in the workspace.
+constexpr size_t kSmemCeiling = 200 * 1024;
+constexpr size_t kProfileSmemLimit = kSmemCeiling;
+constexpr size_t kValidateSmemLimit = kSmemCeiling;
+constexpr size_t kPlanSmemLimit = kSmemCeiling;
+
+// Raises the kernel's dynamic shared memory ceiling once per device.
+cudaError_t set_smem_limit(const void* func, size_t bytes);
+
+// Alignment of every workspace slice.
+constexpr size_t kAlign = 256;
+__host__ __device__ constexpr size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+cudaError_t launch_live_profile(const mp_batch& bt, int64_t* profile, int64_t* peak_lb, int32_t* status,
+                                cudaStream_t stream);
+
+size_t validate_workspace_bytes(const mp_batch& bt);
+cudaError_t launch_validate(const mp_batch& bt, const int64_t* offsets, int32_t* verdict, int32_t* conflict,
+                            int32_t* status, void* workspace, cudaStream_t stream);
+
+cudaError_t launch_peak(const mp_batch& bt, const int64_t* offsets, int64_t* plan_peak, int32_t* status,
+                        cudaStream_t stream);
+
+// Largest max_tensors mp_plan_greedy_by_size accepts (per-trace counts are
+// packed with a 2-bit tier tag into one int32).
+constexpr int32_t kPlanMaxTensors = (1 << 28) - 1;
+size_t plan_workspace_bytes(const mp_batch& bt);
+cudaError_t launch_plan(const mp_batch& bt, int32_t policy, int64_t* offsets, int64_t* plan_peak,
+                        int32_t* status, void* workspace, cudaStream_t stream);
+
+}  // namespace mp

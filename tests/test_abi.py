@@ -1,0 +1,100 @@
+"""The C ABI library: builds, loads, exports every declared symbol, and rejects
+bad host-side arguments before touching the GPU (so these run without one)."""
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+
+from paper_2203_00448_gb300 import _lib, build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "memplan.h")
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(mp_[a-z_]+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return _lib.load()
+
+
+def test_header_and_binding_agree():
+    assert declared_functions() == sorted(_lib.EXPORTS)
+
+
+def test_every_declared_symbol_exported(lib):
+    out = subprocess.run(["nm", "-D", "--defined-only", build.LIB_PATH], capture_output=True, text=True,
+                         check=True).stdout
+    exported = set(re.findall(r"\s(mp_\w+)$", out, flags=re.M))
+    for name in declared_functions():
+        assert name in exported, name
+        assert getattr(lib, name) is not None
+    # nothing else leaks out under the mp_ prefix
+    assert exported == set(declared_functions())
+
+
+def test_status_strings(lib):
+    assert lib.mp_abi_version() == 1
+    names = [lib.mp_status_string(k).decode() for k in range(7)]
+    assert names == ["MP_OK", "MP_EINVAL", "MP_EOVERFLOW", "MP_ECUDA", "MP_ETIMEOUT", "MP_ENOMEM", "MP_EINTERNAL"]
+    assert lib.mp_status_string(99).decode() == "MP_UNKNOWN"
+
+
+def _batch(**kw):
+    # Fake device addresses: every call below must fail its host-side checks
+    # before any CUDA call could dereference them.
+    b = _lib.MpBatch(4, 16, 16, 0, 40, 40, 0x1000, 0x2000, 0x3000, 0x4000, 0x5000, 0x6000)
+    for k, v in kw.items():
+        setattr(b, k, v)
+    return b
+
+
+def test_host_argument_errors(lib):
+    P = 0x10000
+    EINVAL, ENOMEM = _lib.EINVAL, _lib.ENOMEM
+    assert lib.mp_live_profile(None, P, P, P, None) == EINVAL
+    for bad in (dict(n_traces=-1), dict(reserved0=1), dict(max_steps=-2), dict(n_tensors=-1),
+                dict(trace_ptr=None), dict(size_bytes=0x6004), dict(alloc_step=0x4002)):
+        b = _batch(**bad)
+        assert lib.mp_live_profile(ctypes.byref(b), P, P, P, None) == EINVAL, bad
+        assert lib.mp_peak(ctypes.byref(b), P, P, P, None) == EINVAL, bad
+    b = _batch(profile_ptr=None)
+    assert lib.mp_live_profile(ctypes.byref(b), P, P, P, None) == EINVAL
+    b = _batch()
+    assert lib.mp_live_profile(ctypes.byref(b), None, P, P, None) == EINVAL   # profile output missing
+    assert lib.mp_live_profile(ctypes.byref(b), P + 4, P, P, None) == EINVAL  # misaligned int64
+    assert lib.mp_plan_greedy_by_size(ctypes.byref(b), 7, P, P, P, P, 1 << 30, None) == EINVAL  # policy
+    need = lib.mp_plan_workspace_bytes(ctypes.byref(b))
+    assert need > 0
+    assert lib.mp_plan_greedy_by_size(ctypes.byref(b), 0, P, P, P, P, need - 1, None) == ENOMEM
+    assert lib.mp_plan_greedy_by_size(ctypes.byref(b), 0, P, P, P, None, need, None) == EINVAL
+    assert lib.mp_plan_greedy_by_size(ctypes.byref(b), 0, P, P, P, P + 8, need, None) == EINVAL  # alignment
+    assert lib.mp_validate_plan(ctypes.byref(b), P, None, P, P, P, 1 << 30, None) == EINVAL
+    assert lib.mp_validate_plan(ctypes.byref(b), P, P, P + 2, P, P, 1 << 30, None) == EINVAL
+
+
+def test_workspace_sizes(lib):
+    b = _batch(n_traces=0)
+    assert lib.mp_plan_workspace_bytes(ctypes.byref(b)) == 0
+    assert lib.mp_validate_workspace_bytes(ctypes.byref(b)) == 0
+    small = _batch(n_traces=4096, max_tensors=512, max_steps=1024)
+    assert lib.mp_validate_workspace_bytes(ctypes.byref(small)) == 0  # fits shared memory
+    big = _batch(n_traces=1, max_tensors=20000, max_steps=10000)
+    assert lib.mp_validate_workspace_bytes(ctypes.byref(big)) > 0
+    assert lib.mp_plan_workspace_bytes(ctypes.byref(big)) > lib.mp_plan_workspace_bytes(ctypes.byref(_batch(n_traces=1, max_tensors=200, max_steps=100)))
+
+
+def test_product_path_never_touches_the_oracle():
+    pkg = os.path.join(ROOT, "paper_2203_00448_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        for fn in files:
+            if fn.endswith((".py", ".cu", ".cuh", ".h")):
+                src = open(os.path.join(dirpath, fn)).read()
+                assert not re.search(r"\bimport\s+oracle\b|\bfrom\s+oracle\b|liboracle|oracle\.h", src), fn

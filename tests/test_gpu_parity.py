@@ -1,0 +1,224 @@
+"""GPU path vs CPU oracle, bit-exact (all integer work: tolerance 0).
+
+Every call goes through the C ABI (libmemplan.so) via the package binding.
+Covers the five workloads at full size in the launch configuration the bench
+uses, random ragged batches, shapes that force each placement tier and the
+workspace (global-memory) variants, empty traces, planted plan conflicts and
+every per-trace error code.
+"""
+import functools
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import tracegen as tg
+
+pytestmark = pytest.mark.gpu
+
+POLICIES = (("first", oracle.FIT_FIRST), ("best", oracle.FIT_BEST))
+
+
+def gpu_run(ts, policy):
+    import paper_2203_00448_gb300 as mp
+
+    db = mp.DeviceBatch.from_host(ts, "cuda")
+    res = mp.run_path(db, policy)
+    pk2, st_pk = mp.peak(db, res.offsets)
+    torch.cuda.synchronize()
+    h = lambda t: t.cpu().numpy()
+    return dict(profile=h(res.profile), peak_lb=h(res.peak_lb), offsets=h(res.offsets), plan_peak=h(res.plan_peak),
+                verdict=h(res.verdict), conflict=h(res.conflict), st=h(res.status), peak=h(pk2), st_peak=h(st_pk))
+
+
+def oracle_run(ts, pol):
+    prof, lb, st_p = oracle.live_profile(ts)
+    off, pk, st_g = oracle.plan_greedy_by_size(ts, pol)
+    v, c, st_v = oracle.validate_plan(ts, off)
+    pk2, st_pk = oracle.peak(ts, off)
+    return dict(profile=prof, peak_lb=lb, offsets=off, plan_peak=pk, verdict=v, conflict=c,
+                st=np.stack([st_p, st_g, st_v]), peak=pk2, st_peak=st_pk)
+
+
+@functools.lru_cache(maxsize=None)
+def config_oracle(k, pol):
+    return oracle_run(tg.config(k), pol)
+
+
+def assert_parity(ts, g, o):
+    assert np.array_equal(g["st"], o["st"]), "trace status differs"
+    ok = (o["st"] == 0).all(axis=0)
+    prof_ok = o["st"][0] == 0
+    for b in np.nonzero(prof_ok)[0]:
+        lo, hi = ts.profile_ptr[b], ts.profile_ptr[b + 1]
+        assert np.array_equal(g["profile"][lo:hi], o["profile"][lo:hi]), f"profile of trace {b}"
+    assert np.array_equal(g["peak_lb"][prof_ok], o["peak_lb"][prof_ok])
+    plan_ok = o["st"][1] == 0
+    for b in np.nonzero(plan_ok)[0]:
+        lo, hi = ts.trace_ptr[b], ts.trace_ptr[b + 1]
+        assert np.array_equal(g["offsets"][lo:hi], o["offsets"][lo:hi]), f"offsets of trace {b}"
+    assert np.array_equal(g["plan_peak"][plan_ok], o["plan_peak"][plan_ok])
+    assert np.array_equal(g["verdict"][ok], o["verdict"][ok])
+    assert np.array_equal(g["conflict"][ok], o["conflict"][ok])
+    assert np.array_equal(g["st_peak"], o["st_peak"])
+    assert np.array_equal(g["peak"][ok], o["peak"][ok])
+
+
+@pytest.mark.parametrize("name,pol", POLICIES)
+@pytest.mark.parametrize("k", range(5))
+def test_workload_parity(cuda_lib, k, name, pol):
+    ts = tg.config(k)
+    g = gpu_run(ts, name)
+    o = config_oracle(k, pol)
+    assert (o["st"] == 0).all() and (o["verdict"] == 1).all()
+    assert_parity(ts, g, o)
+
+
+def test_determinism(cuda_lib):
+    ts = tg.config(4)
+    a, b = gpu_run(ts, "best"), gpu_run(ts, "best")
+    for key in a:
+        assert np.array_equal(a[key], b[key]), key
+
+
+@pytest.mark.parametrize("name,pol", POLICIES)
+def test_random_ragged_batches(cuda_lib, name, pol):
+    for seed, n_max, T_max, smax in ((1, 40, 30, 64), (2, 200, 300, 1 << 20), (3, 120, 12, 8), (4, 300, 2000, 1 << 30)):
+        ts = tg.random_small(seed, 300, n_max, T_max, smax)
+        assert_parity(ts, gpu_run(ts, name), oracle_run(ts, pol))
+
+
+@pytest.mark.parametrize("name,pol", POLICIES)
+def test_all_tiers_shared_memory_path(cuda_lib, name, pol):
+    """Cliques and long-lived tensors: predecessor counts from 0 to ~n cover the
+    thread, warp and CTA placement tiers inside one CTA."""
+    rng = np.random.default_rng(100)
+    traces = []
+    for n in (1, 9, 33, 64, 150, 200):
+        T = 50
+        a = rng.integers(0, 10, size=n)
+        f = rng.integers(40, 51, size=n)
+        s = rng.integers(1, 4, size=n) * 64  # many equal sizes: exercises the tie-break
+        traces.append((T, a, f, s))
+        a2 = rng.integers(0, T, size=n)
+        f2 = np.minimum(a2 + rng.integers(1, 60, size=n), T)
+        traces.append((T, a2, f2, rng.integers(1, 5000, size=n)))
+    ts = tg.from_arrays(traces)
+    assert_parity(ts, gpu_run(ts, name), oracle_run(ts, pol))
+
+
+@pytest.mark.parametrize("name,pol", POLICIES)
+def test_global_memory_path(cuda_lib, name, pol):
+    """A trace too large for shared memory runs on the workspace variant; the
+    long tensors spanning ~17,000 short ones exceed the warp enumeration limit."""
+    rng = np.random.default_rng(7)
+    n_short, T = 17000, 9000
+    a = rng.integers(0, T, size=n_short)
+    f = np.minimum(a + 1 + rng.geometric(0.5, size=n_short) - 1, T)
+    s = rng.integers(1, 1 << 16, size=n_short)
+    la = np.array([0, 0, 100, 4000]); lf = np.array([T, T, 8000, 8999])
+    ls = np.array([1 << 20, 64, 5000, 70000])
+    ts = tg.from_arrays([(T, np.concatenate([a, la]), np.concatenate([f, lf]), np.concatenate([s, ls]))])
+    assert_parity(ts, gpu_run(ts, name), oracle_run(ts, pol))
+
+
+def test_empty_and_degenerate(cuda_lib):
+    ts = tg.from_tuples([(0, []), (5, []), (1, [(0, 1, 1)]), (3, [(0, 3, 7), (0, 3, 7), (1, 2, 7)]),
+                         (4, [(0, 4, 2 ** 40), (0, 4, 2 ** 40)])])
+    for name, pol in POLICIES:
+        assert_parity(ts, gpu_run(ts, name), oracle_run(ts, pol))
+
+
+def test_zero_traces(cuda_lib):
+    import paper_2203_00448_gb300 as mp
+
+    ts = tg.from_tuples([])
+    db = mp.DeviceBatch.from_host(ts, "cuda")
+    res = mp.run_path(db, "first")
+    torch.cuda.synchronize()
+    assert res.offsets.numel() == 0 and res.verdict.numel() == 0
+
+
+def test_error_codes(cuda_lib):
+    traces = [
+        (4, [(-1, 2, 8)]),                       # alloc < 0
+        (4, [(2, 2, 8)]),                        # free <= alloc
+        (4, [(1, 5, 8)]),                        # free > T
+        (4, [(0, 1, 0)]),                        # size <= 0
+        (4, [(0, 1, 2 ** 62), (0, 2, 2 ** 62)]),  # sizes overflow int64
+        (4, [(0, 1, 2 ** 62), (0, 1, -5)]),       # EINVAL wins
+        (6, [(0, 3, 64), (1, 4, 32)]),           # fine
+    ]
+    ts = tg.from_tuples(traces)
+    for name, pol in POLICIES:
+        g, o = gpu_run(ts, name), oracle_run(ts, pol)
+        assert o["st"][1].tolist() == [1, 1, 1, 1, 2, 1, 0]
+        assert_parity(ts, g, o)
+
+
+def test_declared_bounds_and_csr_checked(cuda_lib):
+    """Traces breaking the host-declared bounds or the CSR are rejected per trace."""
+    import paper_2203_00448_gb300 as mp
+
+    ts = tg.from_tuples([(4, [(0, 2, 8), (1, 3, 8), (0, 4, 8)]), (3, [(0, 3, 5)])])
+    db = mp.DeviceBatch.from_host(ts, "cuda")
+    db.max_tensors = 2  # trace 0 has 3 tensors
+    _, _, st = mp.plan_greedy_by_size(db)
+    _, _, st2 = mp.validate_plan(db, torch.zeros(ts.n_tensors, dtype=torch.int64, device="cuda"))
+    assert st.tolist() == [1, 0] and st2.tolist() == [1, 0]
+    db = mp.DeviceBatch.from_host(ts, "cuda")
+    db.max_steps = 3
+    _, _, st = mp.live_profile(db)
+    assert st.tolist() == [1, 0]
+    db = mp.DeviceBatch.from_host(ts, "cuda")
+    db.profile_ptr[1] = 3  # trace 0 claims 3 profile entries but T = 4
+    _, _, st = mp.live_profile(db)
+    assert st.tolist() == [1, 1]
+    db = mp.DeviceBatch.from_host(ts, "cuda")
+    db.trace_ptr[1] = 5  # beyond n_tensors = 4
+    _, _, st = mp.plan_greedy_by_size(db)
+    assert st.tolist() == [1, 1]
+
+
+def test_validator_on_planted_conflicts(cuda_lib):
+    import paper_2203_00448_gb300 as mp
+
+    ts = tg.config(2).select(range(0, 4096, 8))
+    off, _, _ = oracle.plan_greedy_by_size(ts, oracle.FIT_FIRST)
+    rng = np.random.default_rng(3)
+    bad = off.copy()
+    for b in range(ts.n_traces):
+        lo, hi = ts.trace_ptr[b], ts.trace_ptr[b + 1]
+        if b % 3 == 0:
+            continue  # leave some traces valid
+        i, j = rng.integers(lo, hi, size=2)
+        bad[j] = bad[i] + (rng.integers(0, 3) * 64)
+    bad[ts.trace_ptr[5]] = -64  # one trace with a negative offset
+    db = mp.DeviceBatch.from_host(ts, "cuda")
+    v, c, st = mp.validate_plan(db, torch.as_tensor(bad, device="cuda"))
+    pk, st_pk = mp.peak(db, torch.as_tensor(bad, device="cuda"))
+    ov, oc, ost = oracle.validate_plan(ts, bad)
+    opk, opst = oracle.peak(ts, bad)
+    assert np.array_equal(st.cpu().numpy(), ost) and np.array_equal(st_pk.cpu().numpy(), opst)
+    okm = ost == 0
+    assert np.array_equal(v.cpu().numpy()[okm], ov[okm])
+    assert np.array_equal(c.cpu().numpy()[okm], oc[okm])
+    assert np.array_equal(pk.cpu().numpy()[okm], opk[okm])
+    assert (ov[okm] == 0).sum() > 100
+
+
+def test_generator_and_oracle_stable_on_this_host(cuda_lib):
+    """The committed oracle summaries reproduce on the GPU host (its CPU may be
+    another architecture), so the parity above compares like with like."""
+    import json
+    import os
+
+    ref = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "config_summaries.json")))
+    for k in (0, 1, 2):
+        c = ref["configs"][k]
+        ts = tg.config(k)
+        assert tg.digest(ts) == c["sha256"]
+        o = config_oracle(k, oracle.FIT_FIRST)
+        assert int(o["offsets"].sum()) == c["first_offsets_sum"]
+        assert int(o["plan_peak"].sum()) == c["first_plan_peak_sum"]
