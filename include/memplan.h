@@ -128,6 +128,32 @@ mp_status mp_plan_greedy_by_size(const mp_batch *batch, mp_fit_policy policy, in
                                  int64_t *plan_peak, int32_t *trace_status, void *workspace,
                                  size_t workspace_bytes, void *stream);
 
+/* Size of the fixed device scratch array behind mp_plan_greedy_by_size_static. */
+#define MP_PLAN_STATIC_SCRATCH_BYTES ((size_t)16 << 20)
+
+/* greedy_by_size without any device allocation by anyone: the same planner
+ * and results as mp_plan_greedy_by_size, but its scratch is a 16 MiB array
+ * that lives inside this library (a file-scope __device__ array), so the
+ * caller passes no workspace.  The paper has no counterpart; this exists for
+ * callers that may not allocate device memory -- a latency-critical serving
+ * path that must not take the allocator's lock, or a plug-in whose host
+ * framework owns the device allocator.  The caller still owns every input
+ * and output buffer.
+ * Limits and rules:
+ * - a batch whose mp_plan_workspace_bytes exceeds MP_PLAN_STATIC_SCRATCH_BYTES
+ *   is rejected with MP_ENOMEM before anything is enqueued;
+ * - the first call on each device (with that device current) looks up the
+ *   array's device address once; make that first call before any stream
+ *   capture;
+ * - all calls share the one array: calls whose kernels overlap on a GPU race
+ *   and must be serialised by the caller; the planner writes every scratch
+ *   byte before reading it, so nothing needs clearing between calls;
+ * - the array occupies device memory on every device that loads this library
+ *   until the process exits.
+ * Other arguments and return codes as for mp_plan_greedy_by_size. */
+mp_status mp_plan_greedy_by_size_static(const mp_batch *batch, mp_fit_policy policy, int64_t *offsets,
+                                        int64_t *plan_peak, int32_t *trace_status, void *stream);
+
 /* Bytes of device workspace mp_validate_plan needs for this batch. */
 size_t mp_validate_workspace_bytes(const mp_batch *batch);
 
