@@ -188,9 +188,10 @@ __device__ __forceinline__ V block_excl_scan(V v, V* red, V* total) {
 }
 
 // In-place exclusive scan of x[0..len) (any memory space) by the whole block,
-// in tiles of blockDim * ITEMS consecutive elements.  red: >= 33 slots.
+// in tiles of blockDim * ITEMS consecutive elements; returns the total.
+// red: >= 33 slots.
 template <typename V, int ITEMS>
-__device__ void block_excl_scan_array(V* x, int64_t len, V* red) {
+__device__ V block_excl_scan_array(V* x, int64_t len, V* red) {
     V carry = 0;
     const int64_t tile = (int64_t)blockDim.x * ITEMS;
     for (int64_t base = 0; base < len; base += tile) {
@@ -212,6 +213,7 @@ __device__ void block_excl_scan_array(V* x, int64_t len, V* red) {
         carry += tot;
         __syncthreads();
     }
+    return carry;
 }
 
 // In-place inclusive scan of x[0..len); returns the block-wide maximum of the

@@ -13,7 +13,7 @@ namespace mp {
 constexpr int kProfileThreads = 256;
 constexpr int kValidateThreads = 256;
 constexpr int kPeakThreads = 256;
-constexpr int kPlanThreadsSmem = 256;    // one CTA per trace, data in shared memory
+constexpr int kPlanThreadsSmem = 128;    // one CTA per trace, data in shared memory
 constexpr int kPlanThreadsGlobal = 1024; // one CTA per trace, data in the workspace
 
 // Largest dynamic shared memory a kernel of this library requests per CTA

@@ -12,26 +12,34 @@
 // overlap i in lifetime never constrains i.  The priority order orients every
 // lifetime-overlap edge, giving a DAG; a tensor can be placed as soon as all
 // of P_i are placed.  One CTA per trace runs Kahn's algorithm over that DAG:
-// PEND[i] = |P_i| counts unplaced predecessors, each round places the whole
-// frontier (tensors in one frontier never overlap each other, so they are
-// independent) and decrements the successors' counters, which pushes the
+// PEND[i] counts unplaced predecessors, each round places the whole frontier
+// (tensors in one frontier never overlap each other, so they are
+// independent) and decrements the successors' counters, which queues the
 // tensors that became ready.  The number of rounds is the DAG's depth, not N.
 // No sort is materialised: the priority order is used only as a comparator.
 //
-// Neighbour enumeration: short-lived tensors (life <= kLongLife) are
-// counting-sorted by alloc step, so the short tensors overlapping i lie in the
-// alloc-step window [alloc_i - Lshort + 1, free_i) (Lshort = longest short
-// lifetime); long-lived tensors sit in a separate list scanned in full.
+// Overlap pairs.  Short-lived tensors (life <= kLongLife) are counting-sorted
+// by alloc step, so each short-short overlapping pair is found once, from the
+// member that starts first (its forward window alloc_j < free_i), and stored
+// in exact per-tensor predecessor / successor lists (count pass, prefix sum,
+// fill pass).  Pairs with a long-lived tensor are found from the long side:
+// the short tensors with alloc in [alloc - Lshort + 1, free) (Lshort = longest
+// short lifetime) and the long tensors after it in the long list.  A short
+// tensor meets its long neighbours by scanning the (small) long list; a long
+// tensor, or every tensor of a trace whose lists exceed their capacity,
+// enumerates its alloc-step window instead.
 //
-// Gap search without sorting: FIRST is the lowest offset o at which
-// [o, o + s_i) meets no predecessor's [off_j, end_j); the answer is 0 or some
-// end_j, so it is the smallest candidate c in {0} U {end_j} that conflicts
-// with no predecessor.  BEST: a gap of the address-ordered scan starts at a
-// candidate c that no predecessor covers (off_j <= c < end_j) and below the
-// top (max end), and has length min{off_j >= c} - c; the smallest length
-// >= s_i wins, the lowest start on ties, else the top.  Both forms are
-// evaluated in parallel over candidates (thread, warp or CTA per tensor,
-// chosen by |P_i| and the enumeration length).
+// Gap search.  FIRST is the lowest offset o at which [o, o + s_i) meets no
+// predecessor [off_j, end_j).  Thread tier: start at o = 0 and jump to the
+// largest end among the predecessors that conflict with [o, o + s_i) until
+// none does (every feasible offset >= o is >= each conflicting end, so the
+// first conflict-free o is the lowest feasible one).  BEST walks the maximal
+// free holes below the top (max end) in address order -- jump off covered
+// points, measure the hole to the next predecessor start -- and keeps the
+// smallest hole that fits, the lowest on ties, else the top.  Warp and CTA
+// tiers (many predecessors) test all candidates {0} U {end_j} in parallel
+// instead: FIRST is the smallest conflict-free candidate; BEST scores each
+// uncovered candidate c below the top by min{off_j >= c} - c.
 #include "common.cuh"
 #include "launch.h"
 
@@ -39,47 +47,64 @@ namespace mp {
 
 namespace {
 
-constexpr int32_t kLongLife = 32;           // lifetimes above this are "long" (performance knob only)
-constexpr int32_t kThreadMaxPred = 4;       // thread tier: at most this many predecessors ...
-constexpr int32_t kThreadMaxRange = 512;    // ... and at most this many enumeration items
-constexpr int32_t kWarpMaxRange = 16384;    // warp tier: enumeration items
-constexpr int32_t kTierShift = 28;             // NPRED = |P_i| | tier << 28 (|P_i| < 2^28)
+constexpr int32_t kLongLife = 32;         // lifetimes above this are "long" (performance knob only)
+constexpr int32_t kListCap = 2;           // list capacity per tensor (pairs), else window mode
+constexpr int32_t kRegPred = 4;           // thread tier keeps up to this many predecessors in registers
+constexpr int32_t kThreadMaxPred = 16;    // thread tier: at most this many predecessors,
+constexpr int32_t kThreadMaxScan = 64;    // ... a predecessor scan of at most this many items
+constexpr int32_t kThreadMaxRange = 512;  // ... and a successor scan of at most this many items
+constexpr int32_t kWarpMaxRange = 16384;  // warp tier: enumeration items
+constexpr int32_t kListedBit = 4;         // INFO: predecessors / successors come from the lists
 enum : int32_t { kTierThread = 0, kTierWarp = 1, kTierCta = 2 };
 
+__host__ __device__ constexpr size_t align16(size_t x) { return (x + 15) & ~size_t(15); }
+
+template <typename I>
 struct PlanLayout {
-    size_t s, off, a, f, bys, longl, pend, npred, queue, aux, bend, total;
+    size_t s, off, pend, pre, sue, aux, bend, a, f, bys, longl, queue, predl, succl, info, total;
     __host__ __device__ PlanLayout(int64_t n, int64_t T) {
         s = 0;
-        off = s + align_up((size_t)n * 8);
-        a = off + align_up((size_t)n * 8);
-        f = a + align_up((size_t)n * 4);
-        bys = f + align_up((size_t)n * 4);
-        longl = bys + align_up((size_t)n * 4);
-        pend = longl + align_up((size_t)n * 4);
-        npred = pend + align_up((size_t)n * 4);
-        queue = npred + align_up((size_t)n * 4);
-        aux = queue + align_up((size_t)n * 4);
-        bend = aux + align_up((size_t)n * 4);
-        total = bend + align_up((size_t)T * 4);
+        off = s + align16((size_t)n * 8);
+        pend = off + align16((size_t)n * 8);
+        pre = pend + align16((size_t)n * 4);
+        sue = pre + align16((size_t)n * 4);
+        aux = sue + align16((size_t)n * 4);
+        bend = aux + align16((size_t)n * 4);
+        a = bend + align16((size_t)T * 4);
+        f = a + align16((size_t)n * sizeof(I));
+        bys = f + align16((size_t)n * sizeof(I));
+        longl = bys + align16((size_t)n * sizeof(I));
+        queue = longl + align16((size_t)n * sizeof(I));
+        predl = queue + align16((size_t)n * sizeof(I));
+        succl = predl + align16((size_t)n * kListCap * sizeof(I));
+        info = succl + align16((size_t)n * kListCap * sizeof(I));
+        total = align_up(info + align16((size_t)n));
     }
 };
 
+template <typename I>
 struct Trace {
     int64_t* S;
     int64_t* OFF;
-    int32_t* A;
-    int32_t* F;
-    int32_t* BYS;    // short tensors sorted by alloc step
-    int32_t* LONGL;  // long tensors, any order
-    int32_t* PEND;   // unplaced predecessors
-    int32_t* NPRED;  // |P_i| | tier << kTierShift, non-negative
-    int32_t* QUEUE;  // topological order as it is discovered
-    int32_t* BEND;   // BEND[t] = number of short tensors with alloc <= t
+    int32_t* PEND;  // unplaced predecessors (|P_i| once the pairs are counted)
+    int32_t* PRE;   // end of i's predecessor list in PREDL (start: PRE[i - 1], or 0)
+    int32_t* SUE;   // end of i's successor list in SUCCL
+    int32_t* AUX;   // per-round tier lists
+    int32_t* BEND;  // BEND[t] = number of short tensors with alloc <= t
+    I* A;
+    I* F;
+    I* BYS;    // short tensors sorted by alloc step
+    I* LONGL;  // long tensors, any order
+    I* QUEUE;  // topological order as it is discovered
+    I* PREDL;  // short predecessors of short tensors, grouped by tensor
+    I* SUCCL;  // short successors of short tensors, grouped by tensor
+    uint8_t* INFO;  // tier | kListedBit
     int32_t n, nlong, lshort;
 };
 
 // j strictly precedes i in priority (size desc, alloc asc, id asc).
-__device__ __forceinline__ bool precedes(const Trace& m, int32_t j, int32_t i) {
+template <typename I>
+__device__ __forceinline__ bool precedes(const Trace<I>& m, int32_t j, int32_t i) {
     const int64_t sj = m.S[j], si = m.S[i];
     if (sj != si) return sj > si;
     const int32_t aj = m.A[j], ai = m.A[i];
@@ -87,14 +112,15 @@ __device__ __forceinline__ bool precedes(const Trace& m, int32_t j, int32_t i) {
     return j < i;
 }
 
-// Enumeration of i's lifetime neighbours: items [0, nshort) are the short
-// tensors with alloc in [alloc_i - lshort + 1, free_i), items
+// Enumeration of all of i's lifetime neighbours: items [0, nshort) are the
+// short tensors with alloc in [alloc_i - lshort + 1, free_i), items
 // [nshort, nshort + nlong) the long list.
 struct Window {
     int32_t ai, fi, p0, nshort, range;
 };
 
-__device__ __forceinline__ Window window_of(const Trace& m, int32_t i) {
+template <typename I>
+__device__ __forceinline__ Window window_of(const Trace<I>& m, int32_t i) {
     Window w;
     w.ai = m.A[i];
     w.fi = m.F[i];
@@ -107,7 +133,8 @@ __device__ __forceinline__ Window window_of(const Trace& m, int32_t i) {
 }
 
 // Item k of i's window: the neighbour's id if it overlaps i in lifetime, else -1.
-__device__ __forceinline__ int32_t neighbour(const Trace& m, int32_t i, const Window& w, int32_t k) {
+template <typename I>
+__device__ __forceinline__ int32_t neighbour(const Trace<I>& m, int32_t i, const Window& w, int32_t k) {
     if (k < w.nshort) {
         const int32_t j = m.BYS[w.p0 + k];  // alloc_j < free_i by the window
         return (j != i && m.F[j] > w.ai) ? j : -1;
@@ -118,19 +145,105 @@ __device__ __forceinline__ int32_t neighbour(const Trace& m, int32_t i, const Wi
 
 // Appends j to the queue; every tensor is pushed exactly once, so the slot is
 // always < n -- the guard only keeps a defect from writing out of bounds.
-__device__ __forceinline__ void enqueue(const Trace& m, int32_t j, int32_t* s_tail) {
+template <typename I>
+__device__ __forceinline__ void enqueue(const Trace<I>& m, int32_t j, int32_t* s_tail) {
     const int32_t pos = atomicAdd(s_tail, 1);
-    if (pos < m.n) m.QUEUE[pos] = j;
+    if (pos < m.n) m.QUEUE[pos] = (I)j;
 }
 
-__device__ __forceinline__ void push_ready(const Trace& m, int32_t j, int32_t* s_tail) {
+template <typename I>
+__device__ __forceinline__ void push_ready(const Trace<I>& m, int32_t j, int32_t* s_tail) {
     if (atomicSub(m.PEND + j, 1) == 1) enqueue(m, j, s_tail);
+}
+
+// Calls fn(j) for every predecessor j of i (listed: short ones from the list,
+// long ones from the long list; else the whole window).
+template <typename I, typename Fn>
+__device__ __forceinline__ void for_each_pred(const Trace<I>& m, int32_t i, bool listed, Fn&& fn) {
+    if (listed) {
+        const int32_t e = m.PRE[i];
+        for (int32_t x = i ? m.PRE[i - 1] : 0; x < e; ++x) fn((int32_t)m.PREDL[x]);
+        const int32_t ai = m.A[i], fi = m.F[i];
+        for (int32_t u = 0; u < m.nlong; ++u) {
+            const int32_t L = m.LONGL[u];
+            if (m.A[L] < fi && m.F[L] > ai && precedes(m, L, i)) fn(L);
+        }
+    } else {
+        const Window w = window_of(m, i);
+        for (int32_t k = 0; k < w.range; ++k) {
+            const int32_t j = neighbour(m, i, w, k);
+            if (j >= 0 && precedes(m, j, i)) fn(j);
+        }
+    }
+}
+
+// Calls fn(j) for every successor j of i.
+template <typename I, typename Fn>
+__device__ __forceinline__ void for_each_succ(const Trace<I>& m, int32_t i, bool listed, Fn&& fn) {
+    if (listed) {
+        const int32_t e = m.SUE[i];
+        for (int32_t x = i ? m.SUE[i - 1] : 0; x < e; ++x) fn((int32_t)m.SUCCL[x]);
+        const int32_t ai = m.A[i], fi = m.F[i];
+        for (int32_t u = 0; u < m.nlong; ++u) {
+            const int32_t L = m.LONGL[u];
+            if (m.A[L] < fi && m.F[L] > ai && precedes(m, i, L)) fn(L);
+        }
+    } else {
+        const Window w = window_of(m, i);
+        for (int32_t k = 0; k < w.range; ++k) {
+            const int32_t j = neighbour(m, i, w, k);
+            if (j >= 0 && precedes(m, i, j)) fn(j);
+        }
+    }
 }
 
 // ------------------------------------------------------------- gap search
 
-// Candidate test over predecessor arrays po/pe of length c (any memory space).
-// FIRST: does [cand, cand + s) avoid every predecessor?
+constexpr int64_t kNone = INT64_MAX;
+
+// FIRST by jumping: `each(fn)` calls fn(off, end) for every predecessor.
+template <typename Each>
+__device__ __forceinline__ int64_t fit_first_scan(int64_t s, Each&& each) {
+    int64_t o = 0;
+    for (;;) {
+        int64_t next = o;
+        each([&](int64_t po, int64_t pe) {
+            if (po < o + s && o < pe && pe > next) next = pe;
+        });
+        if (next == o) return o;
+        o = next;
+    }
+}
+
+// BEST by walking the free holes below the top in address order.
+template <typename Each>
+__device__ __forceinline__ int64_t fit_best_scan(int64_t s, int64_t top, Each&& each) {
+    int64_t c = 0, best_len = kNone, best = top;
+    while (c < top) {
+        for (;;) {  // move c off any predecessor that covers it
+            int64_t next = c;
+            each([&](int64_t po, int64_t pe) {
+                if (po <= c && c < pe && pe > next) next = pe;
+            });
+            if (next == c) break;
+            c = next;
+        }
+        if (c >= top) break;
+        int64_t ns = kNone;  // c is uncovered and below the top: some start lies above it
+        each([&](int64_t po, int64_t) {
+            if (po > c && po < ns) ns = po;
+        });
+        const int64_t len = ns - c;
+        if (len >= s && len < best_len) {
+            best_len = len;
+            best = c;
+        }
+        c = ns;
+    }
+    return best;
+}
+
+// Candidate test over buffered predecessors po/pe of length c (any memory space).
 __device__ __forceinline__ bool span_free(const int64_t* po, const int64_t* pe, int32_t c, int64_t cand,
                                           int64_t s) {
     for (int32_t x = 0; x < c; ++x)
@@ -138,7 +251,6 @@ __device__ __forceinline__ bool span_free(const int64_t* po, const int64_t* pe, 
     return true;
 }
 
-// BEST: is cand uncovered, and how far is the next predecessor start >= cand?
 __device__ __forceinline__ int64_t gap_at(const int64_t* po, const int64_t* pe, int32_t c, int64_t cand) {
     int64_t next = INT64_MAX;
     for (int32_t x = 0; x < c; ++x) {
@@ -149,11 +261,9 @@ __device__ __forceinline__ int64_t gap_at(const int64_t* po, const int64_t* pe, 
     return next - cand;
 }
 
-constexpr int64_t kNone = INT64_MAX;
-
-// Evaluates candidates k = first, first + stride, ... < c + 1 (k = 0 is
-// offset 0, k >= 1 is pe[k - 1]) and returns this participant's best as a
-// (key, val) pair: FIRST -> (cand, cand); BEST -> (gap length, cand).
+// Evaluates candidates k = first, first + stride, ... <= c (k = 0 is offset 0,
+// k >= 1 is pe[k - 1]); returns this participant's best as (key, val):
+// FIRST -> (cand, cand); BEST -> (gap length, cand).
 __device__ __forceinline__ void eval_candidates(int32_t policy, const int64_t* po, const int64_t* pe, int32_t c,
                                                 int64_t s, int64_t top, int32_t first, int32_t stride,
                                                 int64_t& key, int64_t& val) {
@@ -180,70 +290,53 @@ __device__ __forceinline__ int64_t resolve(int32_t policy, int64_t key, int64_t 
 }
 
 // ------------------------------------------------------------- tiers
-// Each tier places one frontier tensor i and, in the same pass over i's
-// neighbours, decrements the pending count of every successor (a neighbour
-// that i precedes).  A successor that reaches zero is queued for the next
+// Each tier places one frontier tensor i and decrements the pending count of
+// every successor.  A successor that reaches zero is queued for the next
 // round, which starts after a barrier, i.e. after OFF[i] is visible.
 
-// Thread tier: at most kThreadMaxPred predecessors, kept in registers.
-__device__ void place_thread(const Trace& m, int32_t policy, int32_t i, int32_t* s_tail) {
-    const Window w = window_of(m, i);
-    int64_t po[kThreadMaxPred], pe[kThreadMaxPred];
+// Thread tier: few predecessors; up to kRegPred are kept in registers, more
+// are re-read from the lists (or the short window) on every pass.
+template <typename I>
+__device__ __forceinline__ void place_thread(const Trace<I>& m, int32_t policy, int32_t i, int32_t* s_tail) {
+    const bool listed = (m.INFO[i] & kListedBit) != 0;
+    const int64_t s = m.S[i];
+    int64_t po[kRegPred], pe[kRegPred];
 #pragma unroll
-    for (int x = 0; x < kThreadMaxPred; ++x) po[x] = pe[x] = 0;
+    for (int x = 0; x < kRegPred; ++x) po[x] = pe[x] = kNone;
     int32_t c = 0;
     int64_t top = 0;
-    for (int32_t k = 0; k < w.range; ++k) {
-        const int32_t j = neighbour(m, i, w, k);
-        if (j < 0) continue;
-        if (!precedes(m, j, i)) {
-            push_ready(m, j, s_tail);
-            continue;
-        }
+    for_each_pred(m, i, listed, [&](int32_t j) {
         const int64_t o = m.OFF[j], e = o + m.S[j];
 #pragma unroll
-        for (int x = 0; x < kThreadMaxPred; ++x)
+        for (int x = 0; x < kRegPred; ++x)
             if (x == c) {
                 po[x] = o;
                 pe[x] = e;
             }
         ++c;
         top = e > top ? e : top;
-    }
-    const int64_t s = m.S[i];
-    int64_t best_key = kNone, best_val = kNone;
+    });
+    int64_t off;
+    if (c <= kRegPred) {
+        auto each = [&](auto&& fn) {
 #pragma unroll
-    for (int k = 0; k <= kThreadMaxPred; ++k) {
-        if (k > c) break;
-        const int64_t cand = k == 0 ? 0 : pe[k - 1];
-        bool ok = true;
-        int64_t next = INT64_MAX;
-#pragma unroll
-        for (int x = 0; x < kThreadMaxPred; ++x) {
-            if (x >= c) break;
-            if (policy == MP_FIT_FIRST) {
-                if (po[x] < cand + s && cand < pe[x]) ok = false;
-            } else {
-                if (po[x] <= cand && cand < pe[x]) ok = false;
-                if (po[x] >= cand && po[x] < next) next = po[x];
-            }
-        }
-        if (!ok) continue;
-        if (policy == MP_FIT_FIRST) {
-            if (cand < best_key) best_key = best_val = cand;
-        } else if (cand < top) {
-            const int64_t len = next - cand;
-            if (len >= s && (len < best_key || (len == best_key && cand < best_val))) {
-                best_key = len;
-                best_val = cand;
-            }
-        }
+            for (int x = 0; x < kRegPred; ++x)
+                if (x < c) fn(po[x], pe[x]);
+        };
+        off = policy == MP_FIT_FIRST ? fit_first_scan(s, each) : fit_best_scan(s, top, each);
+    } else {
+        auto each = [&](auto&& fn) {
+            for_each_pred(m, i, listed, [&](int32_t j) { fn(m.OFF[j], m.OFF[j] + m.S[j]); });
+        };
+        off = policy == MP_FIT_FIRST ? fit_first_scan(s, each) : fit_best_scan(s, top, each);
     }
-    m.OFF[i] = resolve(policy, best_key, best_val, top);
+    m.OFF[i] = off;
+    for_each_succ(m, i, listed, [&](int32_t j) { push_ready(m, j, s_tail); });
 }
 
 // Warp tier: predecessors gathered into this warp's buffer slice (capacity wcap).
-__device__ void place_warp(const Trace& m, int32_t policy, int32_t i, int64_t* bo, int64_t* be, int32_t wcap,
+template <typename I>
+__device__ __forceinline__ void place_warp(const Trace<I>& m, int32_t policy, int32_t i, int64_t* bo, int64_t* be, int32_t wcap,
                            int32_t* s_tail, int32_t* s_err) {
     const int lane = threadIdx.x & 31;
     const Window w = window_of(m, i);
@@ -283,7 +376,8 @@ __device__ void place_warp(const Trace& m, int32_t policy, int32_t i, int64_t* b
 }
 
 // CTA tier: every thread of the block takes part (uniform control flow).
-__device__ void place_cta(const Trace& m, int32_t policy, int32_t i, int64_t* bo, int64_t* be, int32_t cap,
+template <typename I>
+__device__ __forceinline__ void place_cta(const Trace<I>& m, int32_t policy, int32_t i, int64_t* bo, int64_t* be, int32_t cap,
                           int32_t* s_tail, int32_t* s_cnt, unsigned long long* s_top, int32_t* s_err,
                           int64_t* red) {
     const Window w = window_of(m, i);
@@ -320,30 +414,8 @@ __device__ void place_cta(const Trace& m, int32_t policy, int32_t i, int64_t* bo
     __syncthreads();
 }
 
-// Records |P_i| and the tier of tensor i, and seeds the queue with tensors
-// that have no predecessor.
-__device__ __forceinline__ void finish_count(const Trace& m, int32_t i, const Window& w, int32_t cnt, int32_t wcap,
-                                             int32_t* s_tail) {
-    const int32_t tier = (cnt <= kThreadMaxPred && w.range <= kThreadMaxRange) ? kTierThread
-                         : (cnt <= wcap && w.range <= kWarpMaxRange)             ? kTierWarp
-                                                                                 : kTierCta;
-    m.NPRED[i] = cnt | (tier << kTierShift);
-    m.PEND[i] = cnt;
-    if (cnt == 0) enqueue(m, i, s_tail);
-}
-
-__device__ __forceinline__ int32_t count_preds(const Trace& m, int32_t i, const Window& w, int32_t first,
-                                               int32_t stride) {
-    int32_t cnt = 0;
-    for (int32_t k = first; k < w.range; k += stride) {
-        const int32_t j = neighbour(m, i, w, k);
-        cnt += (j >= 0 && precedes(m, j, i)) ? 1 : 0;
-    }
-    return cnt;
-}
-
-template <bool kSmem>
-__global__ void __launch_bounds__(kSmem ? kPlanThreadsSmem : kPlanThreadsGlobal)
+template <typename I, bool kSmem>
+__global__ void __launch_bounds__(kSmem ? kPlanThreadsSmem : kPlanThreadsGlobal, kSmem ? 8 : 1)
 k_plan(mp_batch bt, int32_t policy, int64_t* __restrict__ offsets, int64_t* __restrict__ plan_peak,
        int32_t* __restrict__ status, unsigned char* __restrict__ ws, size_t data_stride, size_t buf_offset,
        size_t buf_stride) {
@@ -358,20 +430,24 @@ k_plan(mp_batch bt, int32_t policy, int64_t* __restrict__ offsets, int64_t* __re
         return;
     }
     const int32_t n = tv.n, T = tv.T;
-    const PlanLayout L(kSmem ? n : bt.max_tensors, kSmem ? T : bt.max_steps);
+    const PlanLayout<I> L(kSmem ? n : bt.max_tensors, kSmem ? T : bt.max_steps);
     unsigned char* base = kSmem ? smem_raw : ws + (size_t)b * data_stride;
-    Trace m;
+    Trace<I> m;
     m.S = reinterpret_cast<int64_t*>(base + L.s);
     m.OFF = reinterpret_cast<int64_t*>(base + L.off);
-    m.A = reinterpret_cast<int32_t*>(base + L.a);
-    m.F = reinterpret_cast<int32_t*>(base + L.f);
-    m.BYS = reinterpret_cast<int32_t*>(base + L.bys);
-    m.LONGL = reinterpret_cast<int32_t*>(base + L.longl);
     m.PEND = reinterpret_cast<int32_t*>(base + L.pend);
-    m.NPRED = reinterpret_cast<int32_t*>(base + L.npred);
-    m.QUEUE = reinterpret_cast<int32_t*>(base + L.queue);
+    m.PRE = reinterpret_cast<int32_t*>(base + L.pre);
+    m.SUE = reinterpret_cast<int32_t*>(base + L.sue);
+    m.AUX = reinterpret_cast<int32_t*>(base + L.aux);
     m.BEND = reinterpret_cast<int32_t*>(base + L.bend);
-    int32_t* AUX = reinterpret_cast<int32_t*>(base + L.aux);  // deferred (warp / CTA) tensors
+    m.A = reinterpret_cast<I*>(base + L.a);
+    m.F = reinterpret_cast<I*>(base + L.f);
+    m.BYS = reinterpret_cast<I*>(base + L.bys);
+    m.LONGL = reinterpret_cast<I*>(base + L.longl);
+    m.QUEUE = reinterpret_cast<I*>(base + L.queue);
+    m.PREDL = reinterpret_cast<I*>(base + L.predl);
+    m.SUCCL = reinterpret_cast<I*>(base + L.succl);
+    m.INFO = reinterpret_cast<uint8_t*>(base + L.info);
     m.n = n;
     const int32_t cap = bt.max_tensors;
     int64_t* bo = reinterpret_cast<int64_t*>(ws + buf_offset + (size_t)b * buf_stride);
@@ -381,6 +457,11 @@ k_plan(mp_batch bt, int32_t policy, int64_t* __restrict__ offsets, int64_t* __re
 
     // ---- phase 1: load, check, classify short / long
     for (int t = threadIdx.x; t < T; t += blockDim.x) m.BEND[t] = 0;
+    for (int k = threadIdx.x; k < n; k += blockDim.x) {
+        m.PEND[k] = 0;
+        m.PRE[k] = 0;
+        m.SUE[k] = 0;
+    }
     if (threadIdx.x == 0) {
         s_nlong = 0;
         s_lshort = 0;
@@ -403,12 +484,12 @@ k_plan(mp_batch bt, int32_t policy, int64_t* __restrict__ offsets, int64_t* __re
             continue;
         }
         sum = sat_add(sum, (uint64_t)s);
-        m.A[k] = a;
-        m.F[k] = f;
+        m.A[k] = (I)a;
+        m.F[k] = (I)f;
         m.S[k] = s;
         const int32_t life = f - a;
         if (life > kLongLife) {
-            m.LONGL[atomicAdd(&s_nlong, 1)] = k;
+            m.LONGL[atomicAdd(&s_nlong, 1)] = (I)k;
         } else {
             atomicAdd(m.BEND + a, 1);
             atomicMax(&s_lshort, life);
@@ -422,49 +503,82 @@ k_plan(mp_batch bt, int32_t policy, int64_t* __restrict__ offsets, int64_t* __re
     }
     m.nlong = s_nlong;
     m.lshort = s_lshort;
+    const int32_t nshort = n - m.nlong;
 
     // ---- phase 2: counting sort of the short tensors by alloc step
     block_excl_scan_array<int32_t, 4>(m.BEND, T, reinterpret_cast<int32_t*>(red));
     for (int k = threadIdx.x; k < n; k += blockDim.x)
-        if (m.F[k] - m.A[k] <= kLongLife) m.BYS[atomicAdd(m.BEND + m.A[k], 1)] = k;
+        if (m.F[k] - m.A[k] <= kLongLife) m.BYS[atomicAdd(m.BEND + m.A[k], 1)] = (I)k;
     __syncthreads();
 
-    // ---- phase 3: |P_i| per tensor, tier, and the first frontier.  Tensors
-    // with long enumeration windows are listed in AUX and counted by a warp
-    // (or by the whole CTA) afterwards.
-    for (int32_t i = threadIdx.x; i < n; i += blockDim.x) {
-        const Window w = window_of(m, i);
-        if (w.range > kThreadMaxRange) {
-            AUX[atomicAdd(&s_nw, 1)] = i;
-            continue;
+    // ---- phase 3: every overlapping pair once.  Short-short pairs from the
+    // earlier-starting member's forward window (one thread per short tensor),
+    // counted, then written into exact lists after a prefix sum; pairs with a
+    // long tensor from the long side (one warp per long tensor), counted only.
+    auto short_pairs = [&](auto&& on_pair) {
+        for (int32_t p = threadIdx.x; p < nshort; p += blockDim.x) {
+            const int32_t i = m.BYS[p];
+            const int32_t stop = m.BEND[m.F[i] - 1];
+            for (int32_t q = p + 1; q < stop; ++q) {
+                const int32_t j = m.BYS[q];
+                if (precedes(m, i, j)) on_pair(i, j);
+                else on_pair(j, i);
+            }
         }
-        finish_count(m, i, w, count_preds(m, i, w, 0, 1), wcap, &s_tail);
+    };
+    short_pairs([&](int32_t hi, int32_t lo) {
+        atomicAdd(m.PRE + lo, 1);
+        atomicAdd(m.SUE + hi, 1);
+    });
+    for (int32_t u = warp; u < m.nlong; u += nwarps) {
+        const int32_t Lt = m.LONGL[u];
+        const Window w = window_of(m, Lt);
+        for (int32_t k = lane; k < w.nshort; k += 32) {
+            const int32_t j = m.BYS[w.p0 + k];
+            if (m.F[j] > w.ai) atomicAdd(m.PEND + (precedes(m, Lt, j) ? j : Lt), 1);
+        }
+        for (int32_t v = u + 1 + lane; v < m.nlong; v += 32) {
+            const int32_t j = m.LONGL[v];
+            if (m.A[j] < w.fi && m.F[j] > w.ai) atomicAdd(m.PEND + (precedes(m, Lt, j) ? j : Lt), 1);
+        }
     }
     __syncthreads();
-    const int32_t naux = s_nw;
-    for (int32_t q = warp; q < naux; q += nwarps) {
-        const int32_t i = AUX[q];
-        const Window w = window_of(m, i);
-        if (w.range > kWarpMaxRange) continue;
-        int32_t cnt = count_preds(m, i, w, lane, 32);
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, o);
-        if (lane == 0) finish_count(m, i, w, cnt, wcap, &s_tail);
+    for (int k = threadIdx.x; k < n; k += blockDim.x) m.PEND[k] += m.PRE[k];
+    __syncthreads();
+    const int32_t n_short_pairs = block_excl_scan_array<int32_t, 4>(m.PRE, n, reinterpret_cast<int32_t*>(red));
+    block_excl_scan_array<int32_t, 4>(m.SUE, n, reinterpret_cast<int32_t*>(red));
+    const bool lists = n_short_pairs <= kListCap * n;
+    if (lists) {
+        short_pairs([&](int32_t hi, int32_t lo) {
+            m.PREDL[atomicAdd(m.PRE + lo, 1)] = (I)hi;
+            m.SUCCL[atomicAdd(m.SUE + hi, 1)] = (I)lo;
+        });
     }
     __syncthreads();
-    for (int32_t q = 0; q < naux; ++q) {
-        const int32_t i = AUX[q];
-        const Window w = window_of(m, i);
-        if (w.range <= kWarpMaxRange) continue;
-        if (threadIdx.x == 0) s_cnt = 0;
-        __syncthreads();
-        atomicAdd(&s_cnt, count_preds(m, i, w, threadIdx.x, blockDim.x));
-        __syncthreads();
-        if (threadIdx.x == 0) finish_count(m, i, w, s_cnt, wcap, &s_tail);
-        __syncthreads();
+
+    // ---- phase 4: tiers and the first frontier
+    for (int32_t i = threadIdx.x; i < n; i += blockDim.x) {
+        const int32_t P = m.PEND[i];
+        const bool listed = lists && (m.F[i] - m.A[i] <= kLongLife);
+        int32_t pred_scan, succ_scan, range = 0;
+        if (listed) {
+            pred_scan = m.PRE[i] - (i ? m.PRE[i - 1] : 0) + m.nlong;
+            succ_scan = m.SUE[i] - (i ? m.SUE[i - 1] : 0) + m.nlong;
+        } else {
+            range = window_of(m, i).range;
+            pred_scan = succ_scan = range;
+        }
+        if (range == 0 && !(P <= kThreadMaxPred && pred_scan <= kThreadMaxScan && succ_scan <= kThreadMaxRange))
+            range = window_of(m, i).range;
+        const int32_t tier =
+            (P <= kThreadMaxPred && pred_scan <= kThreadMaxScan && succ_scan <= kThreadMaxRange) ? kTierThread
+            : (P <= wcap && range <= kWarpMaxRange)                                               ? kTierWarp
+                                                                                                   : kTierCta;
+        m.INFO[i] = (uint8_t)(tier | (listed ? kListedBit : 0));
+        if (P == 0) enqueue(m, i, &s_tail);
     }
 
-    // ---- phase 4: frontier rounds (at most n; each places >= 1 tensor).
+    // ---- phase 5: frontier rounds (at most n; each places >= 1 tensor).
     // Warp-tier tensors of the round are listed at the front of AUX, CTA-tier
     // tensors at the back.
     int32_t qh = 0;
@@ -479,24 +593,25 @@ k_plan(mp_batch bt, int32_t policy, int64_t* __restrict__ offsets, int64_t* __re
         if (qt == qh) break;
         for (int32_t q = qh + threadIdx.x; q < qt; q += blockDim.x) {
             const int32_t i = m.QUEUE[q];
-            const int32_t tier = m.NPRED[i] >> kTierShift;
+            const int32_t tier = m.INFO[i] & 3;
             if (tier == kTierThread) place_thread(m, policy, i, &s_tail);
-            else if (tier == kTierWarp) AUX[atomicAdd(&s_nw, 1)] = i;
-            else AUX[n - 1 - atomicAdd(&s_nc, 1)] = i;
+            else if (tier == kTierWarp) m.AUX[atomicAdd(&s_nw, 1)] = i;
+            else m.AUX[n - 1 - atomicAdd(&s_nc, 1)] = i;
         }
         __syncthreads();
         const int32_t nw = s_nw, nc = s_nc;
         for (int32_t q = warp; q < nw; q += nwarps)
-            place_warp(m, policy, AUX[q], bo + (size_t)warp * wcap, be + (size_t)warp * wcap, wcap, &s_tail, &s_err);
+            place_warp(m, policy, m.AUX[q], bo + (size_t)warp * wcap, be + (size_t)warp * wcap, wcap, &s_tail,
+                       &s_err);
         if (nc > 0) {
             __syncthreads();
             for (int32_t q = 0; q < nc; ++q)
-                place_cta(m, policy, AUX[n - 1 - q], bo, be, cap, &s_tail, &s_cnt, &s_top, &s_err, red);
+                place_cta(m, policy, m.AUX[n - 1 - q], bo, be, cap, &s_tail, &s_cnt, &s_top, &s_err, red);
         }
         qh = qt;
     }
 
-    // ---- phase 5: offsets out, plan peak
+    // ---- phase 6: offsets out, plan peak
     int64_t mx = 0;
     for (int k = threadIdx.x; k < n; k += blockDim.x) {
         const int64_t e = m.OFF[k] + m.S[k];
@@ -511,19 +626,36 @@ k_plan(mp_batch bt, int32_t policy, int64_t* __restrict__ offsets, int64_t* __re
 }
 
 struct PlanGeometry {
-    bool smem;
-    size_t data_stride, buf_offset, buf_stride, workspace;
+    bool smem, narrow;
+    size_t data, data_stride, buf_offset, buf_stride, workspace;
 };
 
+// 16-bit indices when every id and step fits; shared memory when the trace's
+// working set fits under the ceiling, else a workspace slice per trace.
 PlanGeometry plan_geometry(const mp_batch& bt) {
     PlanGeometry g;
-    const size_t data = PlanLayout(bt.max_tensors, bt.max_steps).total;
-    g.smem = data <= kPlanSmemLimit;
-    g.data_stride = g.smem ? 0 : data;
+    g.narrow = bt.max_tensors <= 32767 && bt.max_steps <= 32767;
+    g.data = g.narrow ? PlanLayout<int16_t>(bt.max_tensors, bt.max_steps).total
+                      : PlanLayout<int32_t>(bt.max_tensors, bt.max_steps).total;
+    g.smem = g.data <= kPlanSmemLimit;
+    g.data_stride = g.smem ? 0 : g.data;
     g.buf_offset = (size_t)bt.n_traces * g.data_stride;
     g.buf_stride = align_up((size_t)bt.max_tensors * 16);
     g.workspace = bt.n_traces == 0 ? 0 : g.buf_offset + (size_t)bt.n_traces * g.buf_stride;
     return g;
+}
+
+template <typename I, bool kSmem>
+cudaError_t launch_variant(const mp_batch& bt, const PlanGeometry& g, int32_t policy, int64_t* offsets,
+                           int64_t* plan_peak, int32_t* status, unsigned char* ws, cudaStream_t stream) {
+    const size_t smem = kSmem ? g.data : 0;
+    if (kSmem) {
+        cudaError_t e = set_smem_limit((const void*)k_plan<I, kSmem>, smem);
+        if (e != cudaSuccess) return e;
+    }
+    k_plan<I, kSmem><<<(unsigned)bt.n_traces, kSmem ? kPlanThreadsSmem : kPlanThreadsGlobal, smem, stream>>>(
+        bt, policy, offsets, plan_peak, status, ws, g.data_stride, g.buf_offset, g.buf_stride);
+    return cudaGetLastError();
 }
 
 }  // namespace
@@ -535,17 +667,11 @@ cudaError_t launch_plan(const mp_batch& bt, int32_t policy, int64_t* offsets, in
     if (bt.n_traces == 0) return cudaSuccess;
     const PlanGeometry g = plan_geometry(bt);
     unsigned char* ws = static_cast<unsigned char*>(workspace);
-    if (g.smem) {
-        const size_t smem = PlanLayout(bt.max_tensors, bt.max_steps).total;
-        cudaError_t e = set_smem_limit((const void*)k_plan<true>, smem);
-        if (e != cudaSuccess) return e;
-        k_plan<true><<<(unsigned)bt.n_traces, kPlanThreadsSmem, smem, stream>>>(
-            bt, policy, offsets, plan_peak, status, ws, 0, g.buf_offset, g.buf_stride);
-    } else {
-        k_plan<false><<<(unsigned)bt.n_traces, kPlanThreadsGlobal, 0, stream>>>(
-            bt, policy, offsets, plan_peak, status, ws, g.data_stride, g.buf_offset, g.buf_stride);
-    }
-    return cudaGetLastError();
+    if (g.narrow)
+        return g.smem ? launch_variant<int16_t, true>(bt, g, policy, offsets, plan_peak, status, ws, stream)
+                      : launch_variant<int16_t, false>(bt, g, policy, offsets, plan_peak, status, ws, stream);
+    return g.smem ? launch_variant<int32_t, true>(bt, g, policy, offsets, plan_peak, status, ws, stream)
+                  : launch_variant<int32_t, false>(bt, g, policy, offsets, plan_peak, status, ws, stream);
 }
 
 }  // namespace mp
