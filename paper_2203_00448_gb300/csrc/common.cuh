@@ -58,6 +58,19 @@ __device__ __forceinline__ uint64_t sat_add(uint64_t x, uint64_t y) {
     return (r < x || r > kSatCap) ? kSatCap : r;
 }
 
+// Atomic 64-bit add built from 32-bit shared-memory atomics (64-bit shared
+// atomics are several times slower): add the low word, take its carry from
+// the value it replaced, and add high word + carry only when that is non-zero.
+// Every 64-bit add is split exactly, so once all adds have completed the word
+// holds the exact sum modulo 2^64; intermediate states are not meaningful.
+__device__ __forceinline__ void atomic_add_u64_split(int64_t* word, uint64_t v) {
+    unsigned int* w = reinterpret_cast<unsigned int*>(word);  // little-endian: w[0] low, w[1] high
+    const unsigned int lo = (unsigned int)v, hi = (unsigned int)(v >> 32);
+    const unsigned int old = atomicAdd(w, lo);
+    const unsigned int h = hi + ((unsigned int)(old + lo) < old ? 1u : 0u);
+    if (h) atomicAdd(w + 1, h);
+}
+
 // ------------------------------------------------------------ warp level
 
 __device__ __forceinline__ uint64_t warp_sat_sum(uint64_t v) {
@@ -106,6 +119,27 @@ __device__ __forceinline__ V warp_incl_scan(V v) {
         if (lane >= o) v += w;
     }
     return v;
+}
+
+// Adds a per-thread size sum (each <= 2^63) into two shared 64-bit counters as
+// exact 32-bit halves: one warp-level reduction, then one atomic pair per warp.
+// The block total exceeds INT64_MAX iff hi + (lo >> 32) >= 2^31 afterwards.
+__device__ __forceinline__ void block_add_size_sum(uint64_t sum, unsigned long long* hi,
+                                                   unsigned long long* lo) {
+    unsigned long long h = sum >> 32, l = sum & 0xffffffffull;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        h += __shfl_xor_sync(0xffffffffu, h, o);
+        l += __shfl_xor_sync(0xffffffffu, l, o);
+    }
+    if ((threadIdx.x & 31) == 0 && (h | l)) {
+        atomicAdd(hi, h);
+        atomicAdd(lo, l);
+    }
+}
+
+__device__ __forceinline__ bool size_sum_overflows(unsigned long long hi, unsigned long long lo) {
+    return hi + (lo >> 32) >= (1ull << 31);
 }
 
 // ------------------------------------------------------------ block level

@@ -10,8 +10,8 @@
 
 namespace mp {
 
-constexpr int kProfileThreads = 256;
-constexpr int kValidateThreads = 256;
+constexpr int kProfileThreads = 128;  // four traces per CTA, one warp each
+constexpr int kValidateThreads = 128;
 constexpr int kPeakThreads = 256;
 constexpr int kPlanThreadsSmem = 128;    // one CTA per trace, data in shared memory
 constexpr int kPlanThreadsGlobal = 1024; // one CTA per trace, data in the workspace

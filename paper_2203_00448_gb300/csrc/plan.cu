@@ -6,40 +6,39 @@
 // placed tensors whose lifetimes overlap its own, the first (FIRST) or the
 // smallest fitting (BEST) gap in address order; above them all if none fits.
 //
-// Parallel form used here (exactly the same result).  Tensor i's offset is a
-// function of the offsets of P_i = { j : overlap(i, j), j precedes i in
-// priority } and of nothing else, because a placed tensor that does not
-// overlap i in lifetime never constrains i.  The priority order orients every
-// lifetime-overlap edge, giving a DAG; a tensor can be placed as soon as all
-// of P_i are placed.  One CTA per trace runs Kahn's algorithm over that DAG:
-// PEND[i] counts unplaced predecessors, each round places the whole frontier
-// (tensors in one frontier never overlap each other, so they are
-// independent) and decrements the successors' counters, which queues the
-// tensors that became ready.  The number of rounds is the DAG's depth, not N.
-// No sort is materialised: the priority order is used only as a comparator.
-//
-// Overlap pairs.  Short-lived tensors (life <= kLongLife) are counting-sorted
-// by alloc step, so each short-short overlapping pair is found once, from the
-// member that starts first (its forward window alloc_j < free_i), and stored
-// in exact per-tensor predecessor / successor lists (count pass, prefix sum,
-// fill pass).  Pairs with a long-lived tensor are found from the long side:
-// the short tensors with alloc in [alloc - Lshort + 1, free) (Lshort = longest
-// short lifetime) and the long tensors after it in the long list.  A short
-// tensor meets its long neighbours by scanning the (small) long list; a long
-// tensor, or every tensor of a trace whose lists exceed their capacity,
-// enumerates its alloc-step window instead.
+// Decomposition used here (exactly the same result).  Tensors whose lifetimes
+// are linked by a chain of overlaps form a connected component; a tensor's
+// offset depends only on tensors of its own component, so components are
+// independent.  Sorted by alloc step (a counting sort into packed records),
+// each component is a contiguous run: a new one starts at position p when no
+// earlier tensor is still live at alloc(p) (the running maximum of free steps
+// is <= alloc(p)).  Each component is then placed by the sequential
+// definition itself:
+//   - at most kThreadComp tensors: one thread, entirely in registers (a
+//     sorting network into priority order, then placement one by one);
+//   - at most kWarpComp tensors: one warp, a tensor per lane; each lane counts
+//     the members that precede it (its priority rank), then the warp places
+//     rank 0, 1, ... in turn, every placed lane testing its own tensor as a
+//     predecessor, with single-instruction warp reductions;
+//   - larger: the whole CTA bitonic-sorts the component into priority order,
+//     then places it tensor by tensor with a CTA-wide gather of the
+//     overlapping placed tensors and a CTA-wide gap search.
+// Batches of short-lived traces split into hundreds of tiny components per
+// trace, so nearly all work runs thread- or warp-parallel with no per-tensor
+// barrier.
 //
 // Gap search.  FIRST is the lowest offset o at which [o, o + s_i) meets no
-// predecessor [off_j, end_j).  Thread tier: start at o = 0 and jump to the
+// predecessor [off_j, end_j).  One thread: start at o = 0 and jump to the
 // largest end among the predecessors that conflict with [o, o + s_i) until
 // none does (every feasible offset >= o is >= each conflicting end, so the
 // first conflict-free o is the lowest feasible one).  BEST walks the maximal
-// free holes below the top (max end) in address order -- jump off covered
-// points, measure the hole to the next predecessor start -- and keeps the
-// smallest hole that fits, the lowest on ties, else the top.  Warp and CTA
-// tiers (many predecessors) test all candidates {0} U {end_j} in parallel
-// instead: FIRST is the smallest conflict-free candidate; BEST scores each
-// uncovered candidate c below the top by min{off_j >= c} - c.
+// free holes below the top (max end) in address order and keeps the smallest
+// that fits, the lowest on ties, else the top.  CTA, few predecessors: every
+// candidate in {0} U {end_j} is tested in parallel (FIRST: smallest
+// conflict-free candidate; BEST: uncovered candidates c below the top scored
+// by min{off_j >= c} - c).  CTA, many predecessors: FIRST by the jump method
+// with block reductions; BEST by sorting the predecessors by offset and
+// scanning the running maximum end, which exposes every gap at once.
 #include "common.cuh"
 #include "launch.h"
 
@@ -47,159 +46,54 @@ namespace mp {
 
 namespace {
 
-constexpr int32_t kLongLife = 32;         // lifetimes above this are "long" (performance knob only)
-constexpr int32_t kListCap = 2;           // list capacity per tensor (pairs), else window mode
-constexpr int32_t kRegPred = 4;           // thread tier keeps up to this many predecessors in registers
-constexpr int32_t kThreadMaxPred = 16;    // thread tier: at most this many predecessors,
-constexpr int32_t kThreadMaxScan = 64;    // ... a predecessor scan of at most this many items
-constexpr int32_t kThreadMaxRange = 512;  // ... and a successor scan of at most this many items
-constexpr int32_t kWarpMaxRange = 16384;  // warp tier: enumeration items
-constexpr int32_t kListedBit = 4;         // INFO: predecessors / successors come from the lists
-enum : int32_t { kTierThread = 0, kTierWarp = 1, kTierCta = 2 };
+constexpr int32_t kThreadComp = 4;  // components up to this size: one thread (registers)
+constexpr int32_t kWarpComp = 32;   // ... up to this size: one warp (a tensor per lane); else the CTA
+constexpr int32_t kCandMax = 64;    // CTA tier: up to this many predecessors, test all candidates
+constexpr int64_t kNone = INT64_MAX;
 
 __host__ __device__ constexpr size_t align16(size_t x) { return (x + 15) & ~size_t(15); }
 
+__host__ __device__ inline int64_t pow2_at_least(int64_t x) {
+    int64_t p = 1;
+    while (p < x) p <<= 1;
+    return p;
+}
+
+// A tensor in alloc-step order, and in priority order (with its offset).
+template <typename I>
+struct ARec {
+    int64_t s;
+    I a, f, id, pad;
+};
+template <typename I>
+struct SRec {
+    int64_t s, off;
+    I a, f, id, pad;
+};
+
 template <typename I>
 struct PlanLayout {
-    size_t s, off, pend, pre, sue, aux, bend, a, f, bys, longl, queue, predl, succl, info, total;
+    size_t arec, offid, bend, cst, lst, xl, total;
     __host__ __device__ PlanLayout(int64_t n, int64_t T) {
-        s = 0;
-        off = s + align16((size_t)n * 8);
-        pend = off + align16((size_t)n * 8);
-        pre = pend + align16((size_t)n * 4);
-        sue = pre + align16((size_t)n * 4);
-        aux = sue + align16((size_t)n * 4);
-        bend = aux + align16((size_t)n * 4);
-        a = bend + align16((size_t)T * 4);
-        f = a + align16((size_t)n * sizeof(I));
-        bys = f + align16((size_t)n * sizeof(I));
-        longl = bys + align16((size_t)n * sizeof(I));
-        queue = longl + align16((size_t)n * sizeof(I));
-        predl = queue + align16((size_t)n * sizeof(I));
-        succl = predl + align16((size_t)n * kListCap * sizeof(I));
-        info = succl + align16((size_t)n * kListCap * sizeof(I));
-        total = align_up(info + align16((size_t)n));
+        arec = 0;
+        offid = arec + align16((size_t)n * sizeof(ARec<I>));
+        bend = offid + align16((size_t)n * 8);
+        cst = bend + align16((size_t)T * 4);
+        lst = cst + align16((size_t)(n + 1) * 4);
+        xl = lst + align16((size_t)n * sizeof(I));
+        total = align_up(xl + align16((size_t)n * sizeof(I)));
     }
 };
 
-template <typename I>
-struct Trace {
-    int64_t* S;
-    int64_t* OFF;
-    int32_t* PEND;  // unplaced predecessors (|P_i| once the pairs are counted)
-    int32_t* PRE;   // end of i's predecessor list in PREDL (start: PRE[i - 1], or 0)
-    int32_t* SUE;   // end of i's successor list in SUCCL
-    int32_t* AUX;   // per-round tier lists
-    int32_t* BEND;  // BEND[t] = number of short tensors with alloc <= t
-    I* A;
-    I* F;
-    I* BYS;    // short tensors sorted by alloc step
-    I* LONGL;  // long tensors, any order
-    I* QUEUE;  // topological order as it is discovered
-    I* PREDL;  // short predecessors of short tensors, grouped by tensor
-    I* SUCCL;  // short successors of short tensors, grouped by tensor
-    uint8_t* INFO;  // tier | kListedBit
-    int32_t n, nlong, lshort;
-};
-
-// j strictly precedes i in priority (size desc, alloc asc, id asc).
-template <typename I>
-__device__ __forceinline__ bool precedes(const Trace<I>& m, int32_t j, int32_t i) {
-    const int64_t sj = m.S[j], si = m.S[i];
-    if (sj != si) return sj > si;
-    const int32_t aj = m.A[j], ai = m.A[i];
-    if (aj != ai) return aj < ai;
-    return j < i;
-}
-
-// Enumeration of all of i's lifetime neighbours: items [0, nshort) are the
-// short tensors with alloc in [alloc_i - lshort + 1, free_i), items
-// [nshort, nshort + nlong) the long list.
-struct Window {
-    int32_t ai, fi, p0, nshort, range;
-};
-
-template <typename I>
-__device__ __forceinline__ Window window_of(const Trace<I>& m, int32_t i) {
-    Window w;
-    w.ai = m.A[i];
-    w.fi = m.F[i];
-    int32_t lo = w.ai - m.lshort + 1;
-    if (lo < 0) lo = 0;
-    w.p0 = lo > 0 ? m.BEND[lo - 1] : 0;
-    w.nshort = m.BEND[w.fi - 1] - w.p0;
-    w.range = w.nshort + m.nlong;
-    return w;
-}
-
-// Item k of i's window: the neighbour's id if it overlaps i in lifetime, else -1.
-template <typename I>
-__device__ __forceinline__ int32_t neighbour(const Trace<I>& m, int32_t i, const Window& w, int32_t k) {
-    if (k < w.nshort) {
-        const int32_t j = m.BYS[w.p0 + k];  // alloc_j < free_i by the window
-        return (j != i && m.F[j] > w.ai) ? j : -1;
-    }
-    const int32_t j = m.LONGL[k - w.nshort];
-    return (j != i && m.A[j] < w.fi && m.F[j] > w.ai) ? j : -1;
-}
-
-// Appends j to the queue; every tensor is pushed exactly once, so the slot is
-// always < n -- the guard only keeps a defect from writing out of bounds.
-template <typename I>
-__device__ __forceinline__ void enqueue(const Trace<I>& m, int32_t j, int32_t* s_tail) {
-    const int32_t pos = atomicAdd(s_tail, 1);
-    if (pos < m.n) m.QUEUE[pos] = (I)j;
-}
-
-template <typename I>
-__device__ __forceinline__ void push_ready(const Trace<I>& m, int32_t j, int32_t* s_tail) {
-    if (atomicSub(m.PEND + j, 1) == 1) enqueue(m, j, s_tail);
-}
-
-// Calls fn(j) for every predecessor j of i (listed: short ones from the list,
-// long ones from the long list; else the whole window).
-template <typename I, typename Fn>
-__device__ __forceinline__ void for_each_pred(const Trace<I>& m, int32_t i, bool listed, Fn&& fn) {
-    if (listed) {
-        const int32_t e = m.PRE[i];
-        for (int32_t x = i ? m.PRE[i - 1] : 0; x < e; ++x) fn((int32_t)m.PREDL[x]);
-        const int32_t ai = m.A[i], fi = m.F[i];
-        for (int32_t u = 0; u < m.nlong; ++u) {
-            const int32_t L = m.LONGL[u];
-            if (m.A[L] < fi && m.F[L] > ai && precedes(m, L, i)) fn(L);
-        }
-    } else {
-        const Window w = window_of(m, i);
-        for (int32_t k = 0; k < w.range; ++k) {
-            const int32_t j = neighbour(m, i, w, k);
-            if (j >= 0 && precedes(m, j, i)) fn(j);
-        }
-    }
-}
-
-// Calls fn(j) for every successor j of i.
-template <typename I, typename Fn>
-__device__ __forceinline__ void for_each_succ(const Trace<I>& m, int32_t i, bool listed, Fn&& fn) {
-    if (listed) {
-        const int32_t e = m.SUE[i];
-        for (int32_t x = i ? m.SUE[i - 1] : 0; x < e; ++x) fn((int32_t)m.SUCCL[x]);
-        const int32_t ai = m.A[i], fi = m.F[i];
-        for (int32_t u = 0; u < m.nlong; ++u) {
-            const int32_t L = m.LONGL[u];
-            if (m.A[L] < fi && m.F[L] > ai && precedes(m, i, L)) fn(L);
-        }
-    } else {
-        const Window w = window_of(m, i);
-        for (int32_t k = 0; k < w.range; ++k) {
-            const int32_t j = neighbour(m, i, w, k);
-            if (j >= 0 && precedes(m, i, j)) fn(j);
-        }
-    }
+// x strictly precedes y in priority (size desc, alloc asc, id asc).
+template <typename R>
+__device__ __forceinline__ bool precedes(const R& x, const R& y) {
+    if (x.s != y.s) return x.s > y.s;
+    if (x.a != y.a) return x.a < y.a;
+    return x.id < y.id;
 }
 
 // ------------------------------------------------------------- gap search
-
-constexpr int64_t kNone = INT64_MAX;
 
 // FIRST by jumping: `each(fn)` calls fn(off, end) for every predecessor.
 template <typename Each>
@@ -243,186 +137,311 @@ __device__ __forceinline__ int64_t fit_best_scan(int64_t s, int64_t top, Each&& 
     return best;
 }
 
-// Candidate test over buffered predecessors po/pe of length c (any memory space).
-__device__ __forceinline__ bool span_free(const int64_t* po, const int64_t* pe, int32_t c, int64_t cand,
-                                          int64_t s) {
-    for (int32_t x = 0; x < c; ++x)
-        if (po[x] < cand + s && cand < pe[x]) return false;
-    return true;
-}
+// ------------------------------------------------------------- one thread
 
-__device__ __forceinline__ int64_t gap_at(const int64_t* po, const int64_t* pe, int32_t c, int64_t cand) {
-    int64_t next = INT64_MAX;
-    for (int32_t x = 0; x < c; ++x) {
-        const int64_t o = po[x];
-        if (o <= cand && cand < pe[x]) return -1;  // covered: not a gap start
-        if (o >= cand && o < next) next = o;
+// Places the component AR[p0, p0 + c), c <= kThreadComp, in registers; writes
+// offsets by id and returns the largest end.
+template <typename I>
+__device__ int64_t place_thread(const ARec<I>* AR, int32_t p0, int32_t c, int32_t policy, int64_t* OFFID) {
+    int64_t s[kThreadComp], off[kThreadComp];
+    int32_t a[kThreadComp], f[kThreadComp], id[kThreadComp];
+#pragma unroll
+    for (int k = 0; k < kThreadComp; ++k) {
+        if (k < c) {
+            const ARec<I> r = AR[p0 + k];
+            s[k] = r.s;
+            a[k] = r.a;
+            f[k] = r.f;
+            id[k] = r.id;
+        } else {  // sentinel: after every real tensor
+            s[k] = -1;
+            a[k] = f[k] = 0;
+            id[k] = INT32_MAX;
+        }
+        off[k] = 0;
     }
-    return next - cand;
-}
-
-// Evaluates candidates k = first, first + stride, ... <= c (k = 0 is offset 0,
-// k >= 1 is pe[k - 1]); returns this participant's best as (key, val):
-// FIRST -> (cand, cand); BEST -> (gap length, cand).
-__device__ __forceinline__ void eval_candidates(int32_t policy, const int64_t* po, const int64_t* pe, int32_t c,
-                                                int64_t s, int64_t top, int32_t first, int32_t stride,
-                                                int64_t& key, int64_t& val) {
-    key = kNone;
-    val = kNone;
-    for (int32_t k = first; k <= c; k += stride) {
-        const int64_t cand = k == 0 ? 0 : pe[k - 1];
+    auto cx = [&](int x, int y) {  // order x before y by priority
+        const bool swap = s[y] != s[x] ? s[y] > s[x] : (a[y] != a[x] ? a[y] < a[x] : id[y] < id[x]);
+        if (swap) {
+            int64_t t64 = s[x]; s[x] = s[y]; s[y] = t64;
+            int32_t t = a[x]; a[x] = a[y]; a[y] = t;
+            t = f[x]; f[x] = f[y]; f[y] = t;
+            t = id[x]; id[x] = id[y]; id[y] = t;
+        }
+    };
+    cx(0, 1); cx(2, 3); cx(0, 2); cx(1, 3); cx(1, 2);  // sorting network for four
+    int64_t mx = 0;
+#pragma unroll
+    for (int r = 0; r < kThreadComp; ++r) {
+        if (r >= c) break;
+        auto each = [&](auto&& fn) {
+#pragma unroll
+            for (int q = 0; q < kThreadComp; ++q)
+                if (q < r && a[q] < f[r] && a[r] < f[q]) fn(off[q], off[q] + s[q]);
+        };
         if (policy == MP_FIT_FIRST) {
-            if (cand < key && span_free(po, pe, c, cand, s)) key = val = cand;
+            off[r] = fit_first_scan(s[r], each);
         } else {
-            if (cand >= top) continue;
-            const int64_t len = gap_at(po, pe, c, cand);
-            if (len >= s && (len < key || (len == key && cand < val))) {
-                key = len;
-                val = cand;
-            }
+            int64_t top = 0;
+            each([&](int64_t, int64_t pe) { top = pe > top ? pe : top; });
+            off[r] = fit_best_scan(s[r], top, each);
         }
+        OFFID[id[r]] = off[r];
+        mx = off[r] + s[r] > mx ? off[r] + s[r] : mx;
     }
+    return mx;
 }
 
-__device__ __forceinline__ int64_t resolve(int32_t policy, int64_t key, int64_t val, int64_t top) {
-    if (policy == MP_FIT_FIRST) return key;  // offset `top` always fits, so key is finite
-    return key == kNone ? top : val;
+// ------------------------------------------------------------- one warp
+
+// Warp max / min of non-negative int64 values by two 32-bit reductions
+// (high words first, then the low words of the lanes holding the top high word).
+__device__ __forceinline__ int64_t warp_max_nonneg(int64_t v) {
+    const unsigned hi = __reduce_max_sync(0xffffffffu, (unsigned)((uint64_t)v >> 32));
+    const unsigned lo = __reduce_max_sync(0xffffffffu, (unsigned)((uint64_t)v >> 32) == hi ? (unsigned)v : 0u);
+    return (int64_t)(((uint64_t)hi << 32) | lo);
+}
+__device__ __forceinline__ int64_t warp_min_nonneg(int64_t v) {
+    const unsigned hi = __reduce_min_sync(0xffffffffu, (unsigned)((uint64_t)v >> 32));
+    const unsigned lo = __reduce_min_sync(0xffffffffu, (unsigned)((uint64_t)v >> 32) == hi ? (unsigned)v : ~0u);
+    return (int64_t)(((uint64_t)hi << 32) | lo);
 }
 
-// ------------------------------------------------------------- tiers
-// Each tier places one frontier tensor i and decrements the pending count of
-// every successor.  A successor that reaches zero is queued for the next
-// round, which starts after a barrier, i.e. after OFF[i] is visible.
-
-// Thread tier: few predecessors; up to kRegPred are kept in registers, more
-// are re-read from the lists (or the short window) on every pass.
+// Places the component AR[p0, p0 + c), c <= 32, with one warp (a tensor per
+// lane); every lane must call it.  Writes offsets by id; returns the largest end.
 template <typename I>
-__device__ __forceinline__ void place_thread(const Trace<I>& m, int32_t policy, int32_t i, int32_t* s_tail) {
-    const bool listed = (m.INFO[i] & kListedBit) != 0;
-    const int64_t s = m.S[i];
-    int64_t po[kRegPred], pe[kRegPred];
-#pragma unroll
-    for (int x = 0; x < kRegPred; ++x) po[x] = pe[x] = kNone;
-    int32_t c = 0;
-    int64_t top = 0;
-    for_each_pred(m, i, listed, [&](int32_t j) {
-        const int64_t o = m.OFF[j], e = o + m.S[j];
-#pragma unroll
-        for (int x = 0; x < kRegPred; ++x)
-            if (x == c) {
-                po[x] = o;
-                pe[x] = e;
-            }
-        ++c;
-        top = e > top ? e : top;
-    });
-    int64_t off;
-    if (c <= kRegPred) {
-        auto each = [&](auto&& fn) {
-#pragma unroll
-            for (int x = 0; x < kRegPred; ++x)
-                if (x < c) fn(po[x], pe[x]);
-        };
-        off = policy == MP_FIT_FIRST ? fit_first_scan(s, each) : fit_best_scan(s, top, each);
-    } else {
-        auto each = [&](auto&& fn) {
-            for_each_pred(m, i, listed, [&](int32_t j) { fn(m.OFF[j], m.OFF[j] + m.S[j]); });
-        };
-        off = policy == MP_FIT_FIRST ? fit_first_scan(s, each) : fit_best_scan(s, top, each);
-    }
-    m.OFF[i] = off;
-    for_each_succ(m, i, listed, [&](int32_t j) { push_ready(m, j, s_tail); });
-}
-
-// Warp tier: predecessors gathered into this warp's buffer slice (capacity wcap).
-template <typename I>
-__device__ __forceinline__ void place_warp(const Trace<I>& m, int32_t policy, int32_t i, int64_t* bo, int64_t* be, int32_t wcap,
-                           int32_t* s_tail, int32_t* s_err) {
+__device__ int64_t place_warp(const ARec<I>* AR, int32_t p0, int32_t c, int32_t policy, int64_t* OFFID) {
+    const unsigned full = 0xffffffffu;
     const int lane = threadIdx.x & 31;
-    const Window w = window_of(m, i);
-    int32_t cnt = 0;
-    int64_t top = 0;
-    for (int32_t kb = 0; kb < w.range; kb += 32) {
-        const int32_t k = kb + lane;
-        const int32_t j = k < w.range ? neighbour(m, i, w, k) : -1;
-        bool hit = false;
-        if (j >= 0) {
-            hit = precedes(m, j, i);
-            if (!hit) push_ready(m, j, s_tail);
+    const bool act = lane < c;
+    ARec<I> me;
+    if (act) me = AR[p0 + lane];
+    const int64_t s = act ? me.s : 0;
+    const int32_t a = act ? (int32_t)me.a : 0, f = act ? (int32_t)me.f : 0, id = act ? (int32_t)me.id : -1;
+    int rank = 0;  // members that precede this one
+    for (int l = 0; l < c; ++l) {
+        const int64_t sl = __shfl_sync(full, s, l);
+        const int32_t al = __shfl_sync(full, a, l), il = __shfl_sync(full, id, l);
+        if (act && l != lane) rank += (sl != s ? sl > s : (al != a ? al < a : il < id)) ? 1 : 0;
+    }
+    int64_t off = 0, end = 0;
+    bool placed = false;
+    for (int r = 0; r < c; ++r) {
+        const int src = __ffs(__ballot_sync(full, act && rank == r)) - 1;
+        const int32_t ai = __shfl_sync(full, a, src), fi = __shfl_sync(full, f, src);
+        const int64_t si = __shfl_sync(full, s, src);
+        const bool pred = placed && a < fi && ai < f;  // placed: ranks below r
+        int64_t o = 0;
+        if (policy == MP_FIT_FIRST) {
+            for (;;) {
+                const int64_t mx = warp_max_nonneg((pred && off < o + si && o < end) ? end : 0);
+                if (mx <= o) break;
+                o = mx;
+            }
+        } else {
+            const int64_t top = warp_max_nonneg(pred ? end : 0);
+            int64_t cc = 0, best_len = kNone;
+            o = top;
+            while (cc < top) {
+                for (;;) {  // move cc off any predecessor that covers it
+                    const int64_t mx = warp_max_nonneg((pred && off <= cc && cc < end) ? end : 0);
+                    if (mx <= cc) break;
+                    cc = mx;
+                }
+                if (cc >= top) break;
+                const int64_t ns = warp_min_nonneg((pred && off > cc) ? off : kNone);
+                const int64_t len = ns - cc;
+                if (len >= si && len < best_len) {
+                    best_len = len;
+                    o = cc;
+                }
+                cc = ns;
+            }
         }
-        const unsigned mask = __ballot_sync(0xffffffffu, hit);
-        if (hit) {
-            const int32_t pos = cnt + __popc(mask & ((1u << lane) - 1u));
-            const int64_t o = m.OFF[j], e = o + m.S[j];
-            if (pos < wcap) {
+        if (lane == src) {
+            off = o;
+            end = o + si;
+            placed = true;
+        }
+    }
+    if (act) OFFID[id] = off;
+    return warp_max_nonneg(act ? end : 0);
+}
+
+// ------------------------------------------------------------- whole CTA
+
+// In-place bitonic sort of keys[0, len) (len a power of two) by `before`;
+// every thread of the block must call it.
+template <typename K, typename Before>
+__device__ void block_bitonic_sort(K* keys, int32_t len, Before&& before) {
+    for (int32_t k = 2; k <= len; k <<= 1) {
+        for (int32_t j = k >> 1; j > 0; j >>= 1) {
+            for (int32_t t = threadIdx.x; t < (len >> 1); t += blockDim.x) {
+                const int32_t lo = 2 * t - (t & (j - 1));  // index with bit j clear
+                const int32_t hi = lo + j;
+                const bool up = (lo & k) == 0;
+                const K x = keys[lo], y = keys[hi];
+                if (up ? before(y, x) : before(x, y)) {
+                    keys[lo] = y;
+                    keys[hi] = x;
+                }
+            }
+            __syncthreads();
+        }
+    }
+}
+
+// Exclusive prefix maximum (identity 0) of one value per thread; the block
+// maximum is left in *total.  red: >= 33 slots.
+__device__ __forceinline__ int64_t block_excl_max(int64_t v, int64_t* red, int64_t* total) {
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+    int64_t incl = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int64_t u = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl = u > incl ? u : incl;
+    }
+    if (lane == 31) red[w] = incl;
+    __syncthreads();
+    if (w == 0) {
+        int64_t xi = lane < nw ? red[lane] : 0;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int64_t u = __shfl_up_sync(0xffffffffu, xi, o);
+            if (lane >= o) xi = u > xi ? u : xi;
+        }
+        const int64_t ex = __shfl_up_sync(0xffffffffu, xi, 1);
+        if (lane < nw) red[lane] = lane == 0 ? 0 : ex;
+        if (lane == nw - 1) red[32] = xi;
+    }
+    __syncthreads();
+    const int64_t up = __shfl_up_sync(0xffffffffu, incl, 1);
+    const int64_t wex = red[w];
+    const int64_t r = lane == 0 ? wex : (up > wex ? up : wex);
+    *total = red[32];
+    __syncthreads();
+    return r;
+}
+
+struct CtaScratch {
+    int64_t* red;  // >= 64 slots
+    int32_t* cnt;
+    unsigned long long* top;
+};
+
+// Places the priority-ordered records R[0, c) of one component with the whole
+// CTA.  bo/be: workspace buffers of at least pow2_at_least(c) entries each.
+template <typename I>
+__device__ void place_large(SRec<I>* R, int32_t c, int32_t policy, int64_t* bo, int64_t* be, const CtaScratch& sc) {
+    for (int32_t r = 0; r < c; ++r) {
+        const int64_t s = R[r].s;
+        const int32_t ai = R[r].a, fi = R[r].f;
+        if (threadIdx.x == 0) {
+            *sc.cnt = 0;
+            *sc.top = 0;
+        }
+        __syncthreads();
+        for (int32_t x = threadIdx.x; x < r; x += blockDim.x) {  // placed, lifetime-overlapping
+            if (R[x].a < fi && ai < R[x].f) {
+                const int64_t o = R[x].off, e = o + R[x].s;
+                const int32_t pos = atomicAdd(sc.cnt, 1);
                 bo[pos] = o;
                 be[pos] = e;
+                atomicMax(sc.top, (unsigned long long)e);
             }
-            top = e > top ? e : top;
         }
-        cnt += __popc(mask);
-    }
-    if (cnt > wcap) {
-        if (lane == 0) *s_err = 1;
-        cnt = wcap;
-    }
-    top = warp_max_i64(top);
-    __syncwarp();
-    int64_t key, val;
-    eval_candidates(policy, bo, be, cnt, m.S[i], top, lane, 32, key, val);
-    warp_min_pair(key, val);
-    if (lane == 0) m.OFF[i] = resolve(policy, key, val, top);
-    __syncwarp();
-}
-
-// CTA tier: every thread of the block takes part (uniform control flow).
-template <typename I>
-__device__ __forceinline__ void place_cta(const Trace<I>& m, int32_t policy, int32_t i, int64_t* bo, int64_t* be, int32_t cap,
-                          int32_t* s_tail, int32_t* s_cnt, unsigned long long* s_top, int32_t* s_err,
-                          int64_t* red) {
-    const Window w = window_of(m, i);
-    if (threadIdx.x == 0) {
-        *s_cnt = 0;
-        *s_top = 0;
-    }
-    __syncthreads();
-    for (int32_t k = threadIdx.x; k < w.range; k += blockDim.x) {
-        const int32_t j = neighbour(m, i, w, k);
-        if (j < 0) continue;
-        if (!precedes(m, j, i)) {
-            push_ready(m, j, s_tail);
-            continue;
-        }
-        const int64_t o = m.OFF[j], e = o + m.S[j];
-        const int32_t pos = atomicAdd(s_cnt, 1);
-        if (pos < cap) {
-            bo[pos] = o;
-            be[pos] = e;
+        __syncthreads();
+        const int32_t P = *sc.cnt;
+        const int64_t top = (int64_t)*sc.top;
+        int64_t key = kNone, val = kNone;
+        if (P <= kCandMax) {
+            for (int32_t k = threadIdx.x; k <= P; k += blockDim.x) {
+                const int64_t cand = k == 0 ? 0 : be[k - 1];
+                if (policy == MP_FIT_FIRST) {
+                    bool ok = true;
+                    for (int32_t x = 0; x < P && ok; ++x) ok = !(bo[x] < cand + s && cand < be[x]);
+                    if (ok && cand < key) key = val = cand;
+                } else if (cand < top) {
+                    int64_t next = INT64_MAX;
+                    bool covered = false;
+                    for (int32_t x = 0; x < P && !covered; ++x) {
+                        covered = bo[x] <= cand && cand < be[x];
+                        if (bo[x] >= cand && bo[x] < next) next = bo[x];
+                    }
+                    const int64_t gl = next - cand;
+                    if (!covered && gl >= s && (gl < key || (gl == key && cand < val))) {
+                        key = gl;
+                        val = cand;
+                    }
+                }
+            }
+            block_min_pair(key, val, sc.red);
+        } else if (policy == MP_FIT_FIRST) {
+            int64_t o = 0;
+            for (;;) {
+                int64_t next = o;
+                for (int32_t x = threadIdx.x; x < P; x += blockDim.x)
+                    if (bo[x] < o + s && o < be[x] && be[x] > next) next = be[x];
+                next = block_max_i64(next, sc.red);
+                if (next == o) break;
+                o = next;
+            }
+            key = val = o;
         } else {
-            *s_err = 1;
+            // Sort predecessors by offset, then gap_k = off_(k) - max end of those before k.
+            const int32_t plen = (int32_t)pow2_at_least(P);
+            for (int32_t x = P + threadIdx.x; x < plen; x += blockDim.x) {
+                bo[x] = INT64_MAX;
+                be[x] = INT64_MAX;
+            }
+            __syncthreads();
+            for (int32_t k = 2; k <= plen; k <<= 1) {
+                for (int32_t j = k >> 1; j > 0; j >>= 1) {
+                    for (int32_t t = threadIdx.x; t < (plen >> 1); t += blockDim.x) {
+                        const int32_t lo = 2 * t - (t & (j - 1)), hi = lo + j;
+                        const bool up = (lo & k) == 0;
+                        const int64_t xo = bo[lo], yo = bo[hi];
+                        if (up ? yo < xo : xo < yo) {
+                            const int64_t xe = be[lo];
+                            bo[lo] = yo;
+                            bo[hi] = xo;
+                            be[lo] = be[hi];
+                            be[hi] = xe;
+                        }
+                    }
+                    __syncthreads();
+                }
+            }
+            const int32_t chunk = (P + blockDim.x - 1) / blockDim.x;
+            const int32_t k0 = min(P, (int32_t)threadIdx.x * chunk), k1 = min(P, k0 + chunk);
+            int64_t local = 0;
+            for (int32_t k = k0; k < k1; ++k) local = be[k] > local ? be[k] : local;
+            int64_t total;
+            int64_t prev = block_excl_max(local, sc.red, &total);
+            for (int32_t k = k0; k < k1; ++k) {
+                const int64_t gl = bo[k] - prev;
+                if (gl >= s && (gl < key || (gl == key && prev < val))) {
+                    key = gl;
+                    val = prev;
+                }
+                prev = be[k] > prev ? be[k] : prev;
+            }
+            block_min_pair(key, val, sc.red);
         }
-        atomicMax(s_top, (unsigned long long)e);
+        if (threadIdx.x == 0) R[r].off = (policy == MP_FIT_FIRST) ? key : (key == kNone ? top : val);
+        __syncthreads();
     }
-    __syncthreads();
-    int32_t c = *s_cnt;
-    c = c < cap ? c : cap;
-    const int64_t top = (int64_t)*s_top;
-    int64_t key, val;
-    eval_candidates(policy, bo, be, c, m.S[i], top, threadIdx.x, blockDim.x, key, val);
-    block_min_pair(key, val, red);
-    if (threadIdx.x == 0) m.OFF[i] = resolve(policy, key, val, top);
-    __syncthreads();
 }
 
 template <typename I, bool kSmem>
-__global__ void __launch_bounds__(kSmem ? kPlanThreadsSmem : kPlanThreadsGlobal, kSmem ? 8 : 1)
+__global__ void __launch_bounds__(kSmem ? kPlanThreadsSmem : kPlanThreadsGlobal)
 k_plan(mp_batch bt, int32_t policy, int64_t* __restrict__ offsets, int64_t* __restrict__ plan_peak,
        int32_t* __restrict__ status, unsigned char* __restrict__ ws, size_t data_stride, size_t buf_offset,
        size_t buf_stride) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
-    __shared__ int64_t red[64];
-    __shared__ int32_t s_nlong, s_lshort, s_tail, s_cnt, s_err, s_nw, s_nc;
-    __shared__ unsigned long long s_top;
+    __shared__ int64_t red[72];
+    __shared__ int32_t s_cnt, s_nt, s_nw, s_nx, s_bad;
+    __shared__ unsigned long long s_top, s_hi, s_lo, s_max;
     const int b = blockIdx.x;
     const TraceView tv = load_trace(bt, b, false);
     if (tv.st != MP_OK) {
@@ -432,196 +451,171 @@ k_plan(mp_batch bt, int32_t policy, int64_t* __restrict__ offsets, int64_t* __re
     const int32_t n = tv.n, T = tv.T;
     const PlanLayout<I> L(kSmem ? n : bt.max_tensors, kSmem ? T : bt.max_steps);
     unsigned char* base = kSmem ? smem_raw : ws + (size_t)b * data_stride;
-    Trace<I> m;
-    m.S = reinterpret_cast<int64_t*>(base + L.s);
-    m.OFF = reinterpret_cast<int64_t*>(base + L.off);
-    m.PEND = reinterpret_cast<int32_t*>(base + L.pend);
-    m.PRE = reinterpret_cast<int32_t*>(base + L.pre);
-    m.SUE = reinterpret_cast<int32_t*>(base + L.sue);
-    m.AUX = reinterpret_cast<int32_t*>(base + L.aux);
-    m.BEND = reinterpret_cast<int32_t*>(base + L.bend);
-    m.A = reinterpret_cast<I*>(base + L.a);
-    m.F = reinterpret_cast<I*>(base + L.f);
-    m.BYS = reinterpret_cast<I*>(base + L.bys);
-    m.LONGL = reinterpret_cast<I*>(base + L.longl);
-    m.QUEUE = reinterpret_cast<I*>(base + L.queue);
-    m.PREDL = reinterpret_cast<I*>(base + L.predl);
-    m.SUCCL = reinterpret_cast<I*>(base + L.succl);
-    m.INFO = reinterpret_cast<uint8_t*>(base + L.info);
-    m.n = n;
-    const int32_t cap = bt.max_tensors;
+    ARec<I>* AR = reinterpret_cast<ARec<I>*>(base + L.arec);
+    int64_t* OFFID = reinterpret_cast<int64_t*>(base + L.offid);
+    int32_t* BEND = reinterpret_cast<int32_t*>(base + L.bend);
+    int32_t* CST = reinterpret_cast<int32_t*>(base + L.cst);
+    I* LST = reinterpret_cast<I*>(base + L.lst);  // thread-tier components from the front, warp-tier from the back
+    I* XL = reinterpret_cast<I*>(base + L.xl);    // CTA-tier components
+    // CTA tier workspace: predecessor offsets / ends, then the priority-ordered records
+    const size_t cap2 = (size_t)pow2_at_least(bt.max_tensors > 0 ? bt.max_tensors : 1);
     int64_t* bo = reinterpret_cast<int64_t*>(ws + buf_offset + (size_t)b * buf_stride);
-    int64_t* be = bo + cap;
-    const int nwarps = blockDim.x >> 5, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int32_t wcap = cap / nwarps;
+    int64_t* be = bo + cap2;
+    SRec<I>* SR = reinterpret_cast<SRec<I>*>(be + cap2);
 
-    // ---- phase 1: load, check, classify short / long
-    for (int t = threadIdx.x; t < T; t += blockDim.x) m.BEND[t] = 0;
-    for (int k = threadIdx.x; k < n; k += blockDim.x) {
-        m.PEND[k] = 0;
-        m.PRE[k] = 0;
-        m.SUE[k] = 0;
-    }
+    // ---- load, check, alloc-step histogram
+    for (int t = threadIdx.x; t < T; t += blockDim.x) BEND[t] = 0;
     if (threadIdx.x == 0) {
-        s_nlong = 0;
-        s_lshort = 0;
-        s_tail = 0;
-        s_err = 0;
-        s_nw = 0;
-        s_nc = 0;
+        s_nt = s_nw = s_nx = 0;
+        s_bad = 0;
+        s_hi = s_lo = s_max = 0;
     }
     __syncthreads();
     const int32_t* __restrict__ Ag = bt.alloc_step + tv.lo;
     const int32_t* __restrict__ Fg = bt.free_step + tv.lo;
     const int64_t* __restrict__ Sg = bt.size_bytes + tv.lo;
-    bool bad = false;
+    bool ok = true;
     uint64_t sum = 0;
-    for (int k = threadIdx.x; k < n; k += blockDim.x) {
-        const int32_t a = __ldg(Ag + k), f = __ldg(Fg + k);
-        const int64_t s = __ldg(Sg + k);
+    auto take = [&](int32_t a, int32_t f, int64_t s) {
         if (!tensor_ok(a, f, s, T)) {
-            bad = true;
-            continue;
+            ok = false;
+            return;
         }
         sum = sat_add(sum, (uint64_t)s);
-        m.A[k] = (I)a;
-        m.F[k] = (I)f;
-        m.S[k] = s;
-        const int32_t life = f - a;
-        if (life > kLongLife) {
-            m.LONGL[atomicAdd(&s_nlong, 1)] = (I)k;
-        } else {
-            atomicAdd(m.BEND + a, 1);
-            atomicMax(&s_lshort, life);
+        atomicAdd(BEND + a, 1);
+    };
+    int k0 = 0;
+    if (((reinterpret_cast<uintptr_t>(Ag) | reinterpret_cast<uintptr_t>(Fg) | reinterpret_cast<uintptr_t>(Sg)) &
+         15) == 0) {
+        const int n4 = n >> 2;
+        for (int q = threadIdx.x; q < n4; q += blockDim.x) {
+            const int4 a = __ldg(reinterpret_cast<const int4*>(Ag) + q);
+            const int4 f = __ldg(reinterpret_cast<const int4*>(Fg) + q);
+            const longlong2 s01 = __ldg(reinterpret_cast<const longlong2*>(Sg) + 2 * q);
+            const longlong2 s23 = __ldg(reinterpret_cast<const longlong2*>(Sg) + 2 * q + 1);
+            take(a.x, f.x, s01.x);
+            take(a.y, f.y, s01.y);
+            take(a.z, f.z, s23.x);
+            take(a.w, f.w, s23.y);
         }
+        k0 = n4 << 2;
     }
-    bad = __syncthreads_or(bad);
-    sum = block_sat_sum(sum, reinterpret_cast<uint64_t*>(red));
-    if (bad || sum > (uint64_t)INT64_MAX) {
-        if (threadIdx.x == 0) status[b] = bad ? MP_EINVAL : MP_EOVERFLOW;
+    for (int k = k0 + threadIdx.x; k < n; k += blockDim.x) take(__ldg(Ag + k), __ldg(Fg + k), __ldg(Sg + k));
+    block_add_size_sum(sum, &s_hi, &s_lo);
+    if (!ok) s_bad = 1;
+    __syncthreads();
+    if (s_bad || size_sum_overflows(s_hi, s_lo)) {
+        if (threadIdx.x == 0) status[b] = s_bad ? MP_EINVAL : MP_EOVERFLOW;
         return;
     }
-    m.nlong = s_nlong;
-    m.lshort = s_lshort;
-    const int32_t nshort = n - m.nlong;
 
-    // ---- phase 2: counting sort of the short tensors by alloc step
-    block_excl_scan_array<int32_t, 4>(m.BEND, T, reinterpret_cast<int32_t*>(red));
-    for (int k = threadIdx.x; k < n; k += blockDim.x)
-        if (m.F[k] - m.A[k] <= kLongLife) m.BYS[atomicAdd(m.BEND + m.A[k], 1)] = (I)k;
-    __syncthreads();
-
-    // ---- phase 3: every overlapping pair once.  Short-short pairs from the
-    // earlier-starting member's forward window (one thread per short tensor),
-    // counted, then written into exact lists after a prefix sum; pairs with a
-    // long tensor from the long side (one warp per long tensor), counted only.
-    auto short_pairs = [&](auto&& on_pair) {
-        for (int32_t p = threadIdx.x; p < nshort; p += blockDim.x) {
-            const int32_t i = m.BYS[p];
-            const int32_t stop = m.BEND[m.F[i] - 1];
-            for (int32_t q = p + 1; q < stop; ++q) {
-                const int32_t j = m.BYS[q];
-                if (precedes(m, i, j)) on_pair(i, j);
-                else on_pair(j, i);
-            }
-        }
-    };
-    short_pairs([&](int32_t hi, int32_t lo) {
-        atomicAdd(m.PRE + lo, 1);
-        atomicAdd(m.SUE + hi, 1);
-    });
-    for (int32_t u = warp; u < m.nlong; u += nwarps) {
-        const int32_t Lt = m.LONGL[u];
-        const Window w = window_of(m, Lt);
-        for (int32_t k = lane; k < w.nshort; k += 32) {
-            const int32_t j = m.BYS[w.p0 + k];
-            if (m.F[j] > w.ai) atomicAdd(m.PEND + (precedes(m, Lt, j) ? j : Lt), 1);
-        }
-        for (int32_t v = u + 1 + lane; v < m.nlong; v += 32) {
-            const int32_t j = m.LONGL[v];
-            if (m.A[j] < w.fi && m.F[j] > w.ai) atomicAdd(m.PEND + (precedes(m, Lt, j) ? j : Lt), 1);
-        }
-    }
-    __syncthreads();
-    for (int k = threadIdx.x; k < n; k += blockDim.x) m.PEND[k] += m.PRE[k];
-    __syncthreads();
-    const int32_t n_short_pairs = block_excl_scan_array<int32_t, 4>(m.PRE, n, reinterpret_cast<int32_t*>(red));
-    block_excl_scan_array<int32_t, 4>(m.SUE, n, reinterpret_cast<int32_t*>(red));
-    const bool lists = n_short_pairs <= kListCap * n;
-    if (lists) {
-        short_pairs([&](int32_t hi, int32_t lo) {
-            m.PREDL[atomicAdd(m.PRE + lo, 1)] = (I)hi;
-            m.SUCCL[atomicAdd(m.SUE + hi, 1)] = (I)lo;
-        });
-    }
-    __syncthreads();
-
-    // ---- phase 4: tiers and the first frontier
-    for (int32_t i = threadIdx.x; i < n; i += blockDim.x) {
-        const int32_t P = m.PEND[i];
-        const bool listed = lists && (m.F[i] - m.A[i] <= kLongLife);
-        int32_t pred_scan, succ_scan, range = 0;
-        if (listed) {
-            pred_scan = m.PRE[i] - (i ? m.PRE[i - 1] : 0) + m.nlong;
-            succ_scan = m.SUE[i] - (i ? m.SUE[i - 1] : 0) + m.nlong;
-        } else {
-            range = window_of(m, i).range;
-            pred_scan = succ_scan = range;
-        }
-        if (range == 0 && !(P <= kThreadMaxPred && pred_scan <= kThreadMaxScan && succ_scan <= kThreadMaxRange))
-            range = window_of(m, i).range;
-        const int32_t tier =
-            (P <= kThreadMaxPred && pred_scan <= kThreadMaxScan && succ_scan <= kThreadMaxRange) ? kTierThread
-            : (P <= wcap && range <= kWarpMaxRange)                                               ? kTierWarp
-                                                                                                   : kTierCta;
-        m.INFO[i] = (uint8_t)(tier | (listed ? kListedBit : 0));
-        if (P == 0) enqueue(m, i, &s_tail);
-    }
-
-    // ---- phase 5: frontier rounds (at most n; each places >= 1 tensor).
-    // Warp-tier tensors of the round are listed at the front of AUX, CTA-tier
-    // tensors at the back.
-    int32_t qh = 0;
-    for (;;) {
-        __syncthreads();
-        const int32_t qt = s_tail < n ? s_tail : n;
-        if (threadIdx.x == 0) {
-            s_nw = 0;
-            s_nc = 0;
-        }
-        __syncthreads();
-        if (qt == qh) break;
-        for (int32_t q = qh + threadIdx.x; q < qt; q += blockDim.x) {
-            const int32_t i = m.QUEUE[q];
-            const int32_t tier = m.INFO[i] & 3;
-            if (tier == kTierThread) place_thread(m, policy, i, &s_tail);
-            else if (tier == kTierWarp) m.AUX[atomicAdd(&s_nw, 1)] = i;
-            else m.AUX[n - 1 - atomicAdd(&s_nc, 1)] = i;
-        }
-        __syncthreads();
-        const int32_t nw = s_nw, nc = s_nc;
-        for (int32_t q = warp; q < nw; q += nwarps)
-            place_warp(m, policy, m.AUX[q], bo + (size_t)warp * wcap, be + (size_t)warp * wcap, wcap, &s_tail,
-                       &s_err);
-        if (nc > 0) {
-            __syncthreads();
-            for (int32_t q = 0; q < nc; ++q)
-                place_cta(m, policy, m.AUX[n - 1 - q], bo, be, cap, &s_tail, &s_cnt, &s_top, &s_err, red);
-        }
-        qh = qt;
-    }
-
-    // ---- phase 6: offsets out, plan peak
-    int64_t mx = 0;
+    // ---- counting sort into alloc-step records (second read hits the cache)
+    block_excl_scan_array<int32_t, 8>(BEND, T, reinterpret_cast<int32_t*>(red));
     for (int k = threadIdx.x; k < n; k += blockDim.x) {
-        const int64_t e = m.OFF[k] + m.S[k];
-        offsets[tv.lo + k] = m.OFF[k];
-        mx = e > mx ? e : mx;
+        const int32_t a = __ldg(Ag + k);
+        ARec<I> r;
+        r.s = __ldg(Sg + k);
+        r.a = (I)a;
+        r.f = (I)__ldg(Fg + k);
+        r.id = (I)k;
+        r.pad = 0;
+        AR[atomicAdd(BEND + a, 1)] = r;
     }
-    mx = block_max_i64(mx, red);
+    __syncthreads();
+
+    // ---- components: a run starts where no earlier tensor is live any more
+    const int32_t chunk = (n + blockDim.x - 1) / blockDim.x;
+    const int32_t q0 = min(n, (int32_t)threadIdx.x * chunk), q1 = min(n, q0 + chunk);
+    int64_t fmax = 0;
+    for (int32_t p = q0; p < q1; ++p) fmax = max(fmax, (int64_t)AR[p].f);
+    int64_t ftot;
+    const int64_t run0 = block_excl_max(fmax, red, &ftot);
+    int32_t starts = 0;
+    {
+        int64_t run = run0;
+        for (int32_t p = q0; p < q1; ++p) {
+            starts += (p == 0 || run <= AR[p].a) ? 1 : 0;
+            run = max(run, (int64_t)AR[p].f);
+        }
+    }
+    int32_t ncomp;
+    const int32_t first = block_excl_scan<int32_t>(starts, reinterpret_cast<int32_t*>(red), &ncomp);
+    {
+        int64_t run = run0;
+        int32_t idx = first;
+        for (int32_t p = q0; p < q1; ++p) {
+            if (p == 0 || run <= AR[p].a) CST[idx++] = p;
+            run = max(run, (int64_t)AR[p].f);
+        }
+    }
+    if (threadIdx.x == 0) CST[ncomp] = n;
+    __syncthreads();
+    for (int32_t c = threadIdx.x; c < ncomp; c += blockDim.x) {
+        const int32_t sz = CST[c + 1] - CST[c];
+        if (sz <= kThreadComp) LST[atomicAdd(&s_nt, 1)] = (I)c;
+        else if (sz <= kWarpComp) LST[n - 1 - atomicAdd(&s_nw, 1)] = (I)c;
+        else XL[atomicAdd(&s_nx, 1)] = (I)c;
+    }
+    __syncthreads();
+
+    // ---- small and medium components: warps take the medium ones, then
+    // every thread the small ones
+    int64_t mx = 0;
+    {
+        const int32_t nw = s_nw, nt = s_nt, nwarps = blockDim.x >> 5;
+        for (int32_t k = threadIdx.x >> 5; k < nw; k += nwarps) {
+            const int32_t c = LST[n - 1 - k], p0 = CST[c];
+            const int64_t e = place_warp(AR, p0, CST[c + 1] - p0, policy, OFFID);
+            mx = e > mx ? e : mx;
+        }
+        for (int32_t k = threadIdx.x; k < nt; k += blockDim.x) {
+            const int32_t c = LST[k], p0 = CST[c];
+            const int64_t e = place_thread(AR, p0, CST[c + 1] - p0, policy, OFFID);
+            mx = e > mx ? e : mx;
+        }
+    }
+
+    // ---- large components, the whole CTA each
+    const int32_t nx = s_nx;
+    const CtaScratch sc{red, &s_cnt, &s_top};
+    for (int32_t q = 0; q < nx; ++q) {
+        const int32_t c = XL[q], p0 = CST[c], sz = CST[c + 1] - p0;
+        const int32_t len = (int32_t)pow2_at_least(sz);
+        int32_t* idx = reinterpret_cast<int32_t*>(bo);  // the index list lives in bo while sorting
+        for (int32_t x = threadIdx.x; x < len; x += blockDim.x) idx[x] = x < sz ? p0 + x : -1;
+        __syncthreads();
+        block_bitonic_sort(idx, len, [&](int32_t x, int32_t y) {  // sentinels (-1) sort last
+            return y < 0 ? x >= 0 : (x >= 0 && precedes(AR[x], AR[y]));
+        });
+        for (int32_t x = threadIdx.x; x < sz; x += blockDim.x) {
+            const ARec<I> me = AR[idx[x]];
+            SRec<I> out;
+            out.s = me.s;
+            out.off = 0;
+            out.a = me.a;
+            out.f = me.f;
+            out.id = me.id;
+            out.pad = 0;
+            SR[x] = out;
+        }
+        __syncthreads();
+        place_large(SR, sz, policy, bo, be, sc);
+        for (int32_t x = threadIdx.x; x < sz; x += blockDim.x) {
+            const int64_t o = SR[x].off;
+            OFFID[SR[x].id] = o;
+            mx = o + SR[x].s > mx ? o + SR[x].s : mx;
+        }
+        __syncthreads();
+    }
+
+    // ---- offsets out, plan peak
+    mx = warp_max_i64(mx);
+    if ((threadIdx.x & 31) == 0 && mx > 0) atomicMax(&s_max, (unsigned long long)mx);
+    __syncthreads();
+    for (int k = threadIdx.x; k < n; k += blockDim.x) offsets[tv.lo + k] = OFFID[k];
     if (threadIdx.x == 0) {
-        plan_peak[b] = mx;
-        status[b] = (qh != n || s_tail != n || s_err) ? MP_EINTERNAL : MP_OK;
+        plan_peak[b] = (int64_t)s_max;
+        status[b] = MP_OK;
     }
 }
 
@@ -631,16 +625,20 @@ struct PlanGeometry {
 };
 
 // 16-bit indices when every id and step fits; shared memory when the trace's
-// working set fits under the ceiling, else a workspace slice per trace.
+// working set fits under the ceiling, else a workspace slice per trace.  The
+// workspace always holds the CTA tier's buffers (predecessor offsets / ends,
+// the index list of a large component, and its records in priority order),
+// sized for up to max_tensors.
 PlanGeometry plan_geometry(const mp_batch& bt) {
     PlanGeometry g;
-    g.narrow = bt.max_tensors <= 32767 && bt.max_steps <= 32767;
+    g.narrow = bt.max_tensors < 32767 && bt.max_steps <= 32767;
     g.data = g.narrow ? PlanLayout<int16_t>(bt.max_tensors, bt.max_steps).total
                       : PlanLayout<int32_t>(bt.max_tensors, bt.max_steps).total;
     g.smem = g.data <= kPlanSmemLimit;
     g.data_stride = g.smem ? 0 : g.data;
     g.buf_offset = (size_t)bt.n_traces * g.data_stride;
-    g.buf_stride = align_up((size_t)bt.max_tensors * 16);
+    const size_t cap2 = (size_t)pow2_at_least(bt.max_tensors > 0 ? bt.max_tensors : 1);
+    g.buf_stride = align_up(cap2 * 16 + (size_t)bt.max_tensors * (g.narrow ? sizeof(SRec<int16_t>) : sizeof(SRec<int32_t>)));
     g.workspace = bt.n_traces == 0 ? 0 : g.buf_offset + (size_t)bt.n_traces * g.buf_stride;
     return g;
 }

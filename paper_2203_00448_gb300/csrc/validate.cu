@@ -19,26 +19,32 @@ namespace mp {
 
 namespace {
 
+// Per-trace working set: tensors scattered into alloc-step order as packed
+// (offset, end) records with their id and free step, plus the bucket ends.
 struct ValidateLayout {
-    size_t off, end, f, bya, bend, total;
+    size_t rec, id, fp, bend, total;
     __host__ __device__ ValidateLayout(int64_t n, int64_t T) {
-        off = 0;
-        end = off + align_up((size_t)n * 8);
-        f = end + align_up((size_t)n * 8);
-        bya = f + align_up((size_t)n * 4);
-        bend = bya + align_up((size_t)n * 4);
+        rec = 0;
+        id = rec + align_up((size_t)n * 16);
+        fp = id + align_up((size_t)n * 4);
+        bend = fp + align_up((size_t)n * 4);
         total = bend + align_up((size_t)T * 4);
     }
 };
 
+struct ValidateShared {
+    unsigned long long key, sum_hi, sum_lo;
+    int bad, ovf;
+};
+
 template <bool kSmem>
-__global__ void __launch_bounds__(kValidateThreads)
+__global__ void __launch_bounds__(kValidateThreads, kSmem ? 12 : 1)
 k_validate(mp_batch bt, const int64_t* __restrict__ offsets, int32_t* __restrict__ verdict,
            int32_t* __restrict__ conflict, int32_t* __restrict__ status, unsigned char* __restrict__ ws,
            size_t ws_stride) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
-    __shared__ int64_t red[64];
-    __shared__ unsigned long long s_key;
+    __shared__ int32_t red[40];
+    __shared__ ValidateShared sh;
     const int b = blockIdx.x;
     const TraceView tv = load_trace(bt, b, false);
     if (tv.st != MP_OK) {
@@ -48,14 +54,17 @@ k_validate(mp_batch bt, const int64_t* __restrict__ offsets, int32_t* __restrict
     const int32_t n = tv.n, T = tv.T;
     const ValidateLayout L(kSmem ? n : bt.max_tensors, kSmem ? T : bt.max_steps);
     unsigned char* base = kSmem ? smem_raw : ws + (size_t)b * ws_stride;
-    int64_t* OFF = reinterpret_cast<int64_t*>(base + L.off);
-    int64_t* END = reinterpret_cast<int64_t*>(base + L.end);
-    int32_t* F = reinterpret_cast<int32_t*>(base + L.f);
-    int32_t* BYA = reinterpret_cast<int32_t*>(base + L.bya);
+    longlong2* REC = reinterpret_cast<longlong2*>(base + L.rec);
+    int32_t* ID = reinterpret_cast<int32_t*>(base + L.id);
+    int32_t* FP = reinterpret_cast<int32_t*>(base + L.fp);
     int32_t* BEND = reinterpret_cast<int32_t*>(base + L.bend);
 
     for (int t = threadIdx.x; t < T; t += blockDim.x) BEND[t] = 0;
-    if (threadIdx.x == 0) s_key = ~0ull;
+    if (threadIdx.x == 0) {
+        sh.key = ~0ull;
+        sh.sum_hi = sh.sum_lo = 0;
+        sh.bad = sh.ovf = 0;
+    }
     __syncthreads();
 
     const int32_t* __restrict__ Ag = bt.alloc_step + tv.lo;
@@ -64,29 +73,43 @@ k_validate(mp_batch bt, const int64_t* __restrict__ offsets, int32_t* __restrict
     const int64_t* __restrict__ Og = offsets + tv.lo;
     bool bad = false, ovf = false;
     uint64_t sum = 0;
-    for (int k = threadIdx.x; k < n; k += blockDim.x) {
-        const int32_t a = __ldg(Ag + k), f = __ldg(Fg + k);
-        const int64_t s = __ldg(Sg + k), o = __ldg(Og + k);
-        if (!tensor_ok(a, f, s, T) || o < 0) {
+    auto check = [&](int32_t a, int32_t f, int64_t sz, int64_t o) {
+        if (!tensor_ok(a, f, sz, T) || o < 0) {
             bad = true;
-            continue;
+            return;
         }
-        sum = sat_add(sum, (uint64_t)s);
-        if (o > INT64_MAX - s) {
-            ovf = true;
-            continue;
-        }
-        OFF[k] = o;
-        END[k] = o + s;
-        F[k] = f;
+        sum = sat_add(sum, (uint64_t)sz);
+        if (o > INT64_MAX - sz) ovf = true;
         atomicAdd(BEND + a, 1);
+    };
+    const bool vec_in = ((reinterpret_cast<uintptr_t>(Ag) | reinterpret_cast<uintptr_t>(Fg) |
+                          reinterpret_cast<uintptr_t>(Sg) | reinterpret_cast<uintptr_t>(Og)) & 15) == 0;
+    int k0 = 0;
+    if (vec_in) {
+        const int n4 = n >> 2;
+        for (int q = threadIdx.x; q < n4; q += blockDim.x) {
+            const int4 a = __ldg(reinterpret_cast<const int4*>(Ag) + q);
+            const int4 f = __ldg(reinterpret_cast<const int4*>(Fg) + q);
+            const longlong2 s01 = __ldg(reinterpret_cast<const longlong2*>(Sg) + 2 * q);
+            const longlong2 s23 = __ldg(reinterpret_cast<const longlong2*>(Sg) + 2 * q + 1);
+            const longlong2 o01 = __ldg(reinterpret_cast<const longlong2*>(Og) + 2 * q);
+            const longlong2 o23 = __ldg(reinterpret_cast<const longlong2*>(Og) + 2 * q + 1);
+            check(a.x, f.x, s01.x, o01.x);
+            check(a.y, f.y, s01.y, o01.y);
+            check(a.z, f.z, s23.x, o23.x);
+            check(a.w, f.w, s23.y, o23.y);
+        }
+        k0 = n4 << 2;
     }
-    bad = __syncthreads_or(bad);
-    ovf = __syncthreads_or(ovf);
-    sum = block_sat_sum(sum, reinterpret_cast<uint64_t*>(red));
-    if (bad || ovf || sum > (uint64_t)INT64_MAX) {
+    for (int k = k0 + threadIdx.x; k < n; k += blockDim.x)
+        check(__ldg(Ag + k), __ldg(Fg + k), __ldg(Sg + k), __ldg(Og + k));
+    block_add_size_sum(sum, &sh.sum_hi, &sh.sum_lo);
+    if (bad) sh.bad = 1;
+    if (ovf) sh.ovf = 1;
+    __syncthreads();
+    if (sh.bad || sh.ovf || size_sum_overflows(sh.sum_hi, sh.sum_lo)) {
         if (threadIdx.x == 0) {
-            status[b] = bad ? MP_EINVAL : MP_EOVERFLOW;
+            status[b] = sh.bad ? MP_EINVAL : MP_EOVERFLOW;
             verdict[b] = 0;
             if (conflict) conflict[2 * b] = conflict[2 * b + 1] = -1;
         }
@@ -94,28 +117,34 @@ k_validate(mp_batch bt, const int64_t* __restrict__ offsets, int32_t* __restrict
     }
     // Counting sort by alloc step: bucket starts, then scatter; afterwards
     // BEND[t] is the end of bucket t (tensors with alloc <= t).
-    block_excl_scan_array<int32_t, 4>(BEND, T, reinterpret_cast<int32_t*>(red));
+    block_excl_scan_array<int32_t, 8>(BEND, T, red);
     for (int k = threadIdx.x; k < n; k += blockDim.x) {
         const int32_t a = __ldg(Ag + k);
-        BYA[atomicAdd(BEND + a, 1)] = k;
+        const int64_t o = __ldg(Og + k);
+        const int32_t pos = atomicAdd(BEND + a, 1);
+        REC[pos] = make_longlong2(o, o + __ldg(Sg + k));
+        ID[pos] = k;
+        FP[pos] = __ldg(Fg + k);
     }
     __syncthreads();
 
+    // Each overlapping pair once, from its earlier member in alloc order.
     for (int p = threadIdx.x; p < n; p += blockDim.x) {
-        const int32_t i = BYA[p];
-        const int32_t stop = BEND[F[i] - 1];
-        const int64_t oi = OFF[i], ei = END[i];
+        const int32_t stop = BEND[FP[p] - 1];
+        if (stop <= p + 1) continue;
+        const longlong2 ri = REC[p];
         for (int q = p + 1; q < stop; ++q) {
-            const int32_t j = BYA[q];
-            if (oi < END[j] && OFF[j] < ei) {
-                const uint32_t lo = (uint32_t)(i < j ? i : j), hi = (uint32_t)(i < j ? j : i);
-                atomicMin(&s_key, ((unsigned long long)lo << 32) | hi);
+            const longlong2 rj = REC[q];
+            if (ri.x < rj.y && rj.x < ri.y) {
+                const uint32_t i = (uint32_t)ID[p], j = (uint32_t)ID[q];
+                const uint32_t lo = i < j ? i : j, hi = i < j ? j : i;
+                atomicMin(&sh.key, ((unsigned long long)lo << 32) | hi);
             }
         }
     }
     __syncthreads();
     if (threadIdx.x == 0) {
-        const unsigned long long key = s_key;
+        const unsigned long long key = sh.key;
         const bool ok = key == ~0ull;
         verdict[b] = ok ? 1 : 0;
         if (conflict) {
