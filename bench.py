@@ -44,7 +44,11 @@ L2_FLUSH_BYTES = 256 << 20
 #           plan_peak 8 B and status 4 B per trace.
 # validate: read alloc/free/size/offset 24 B per tensor and 12 B per trace; write
 #           verdict 4 B, conflict 8 B and status 4 B per trace.
+# fused   : read 16 B per tensor and 20 B per trace; write the profile 8 B per step,
+#           offsets 8 B per tensor, and peak_lb, plan_peak, verdict, conflict and
+#           status (32 B) per trace.
 KERNELS = ("live_profile", "plan_greedy_by_size", "validate_plan")
+FUSED = "plan_and_validate"
 
 
 def algorithmic_bytes(kernel: str, n_tensors: int, n_traces: int, n_steps: int) -> int:
@@ -54,6 +58,8 @@ def algorithmic_bytes(kernel: str, n_tensors: int, n_traces: int, n_steps: int) 
         return 24 * n_tensors + (12 + 12) * n_traces
     if kernel == "validate_plan":
         return 24 * n_tensors + (12 + 16) * n_traces
+    if kernel == FUSED:
+        return 24 * n_tensors + 8 * n_steps + (20 + 32) * n_traces
     raise KeyError(kernel)
 
 
@@ -132,7 +138,7 @@ def ncu_traffic(kernel: str, n_tensors: int):
 
 
 def gpu_id(dev) -> str:
-    """nvidia-smi --id value for a torch device (its UUID, else its index)."""
+    """The device's UUID ("GPU-..."), as NVML and nvidia-smi --id accept it."""
     import torch
 
     uuid = getattr(torch.cuda.get_device_properties(dev), "uuid", None)
@@ -143,45 +149,94 @@ def gpu_id(dev) -> str:
 
 
 class ClockSampler:
-    """nvidia-smi clock / throttle sampling during the timed region."""
+    """SM clock and throttle-reason sampling during the timed region.
 
-    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
-             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
-             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    Reads NVML (read-only queries) from a background thread every millisecond;
+    falls back to `nvidia-smi -lms 100` if NVML cannot be loaded.
+    """
 
-    def __init__(self, gpu_index: int):
-        self.gpu = gpu_index
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown", 0x40: "hw_thermal_slowdown",
+               0x80: "hw_power_brake_slowdown"}
+    SMI_QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+                 "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+                 "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_uuid: str):
+        self.uuid = gpu_uuid
+        self.samples = []  # (sm_mhz, max_mhz, reasons bitmask)
         self.proc = None
+        self.thread = None
+        self.stop = False
+        self.nvml = self._open_nvml()
+
+    def _open_nvml(self):
+        import ctypes
+
+        try:
+            lib = ctypes.CDLL("libnvidia-ml.so.1")
+            if lib.nvmlInit_v2() != 0:
+                return None
+            h = ctypes.c_void_p()
+            if lib.nvmlDeviceGetHandleByUUID(self.uuid.encode(), ctypes.byref(h)) != 0:
+                return None
+            reasons = getattr(lib, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+                lib.nvmlDeviceGetCurrentClocksThrottleReasons
+            return lib, h, reasons
+        except (OSError, AttributeError):
+            return None
+
+    def _poll(self):
+        import ctypes
+
+        lib, h, reasons = self.nvml
+        clk, mx, rs = ctypes.c_uint(), ctypes.c_uint(), ctypes.c_ulonglong()
+        while not self.stop:
+            if lib.nvmlDeviceGetClockInfo(h, 1, ctypes.byref(clk)) == 0 and \
+                    lib.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx)) == 0 and reasons(h, ctypes.byref(rs)) == 0:
+                self.samples.append((clk.value, mx.value, rs.value))
+            time.sleep(0.001)
 
     def __enter__(self):
-        try:
-            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}",
-                                          "--format=csv,noheader,nounits", "-lms", "100"],
-                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
-        except OSError:
-            self.proc = None
+        import threading
+
+        if self.nvml is not None:
+            self.thread = threading.Thread(target=self._poll, daemon=True)
+            self.thread.start()
+        else:
+            try:
+                self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.uuid}", f"--query-gpu={self.SMI_QUERY}",
+                                              "--format=csv,noheader,nounits", "-lms", "100"],
+                                             stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            except OSError:
+                self.proc = None
         return self
 
     def __exit__(self, *exc):
-        self.out = ""
+        if self.thread is not None:
+            self.stop = True
+            self.thread.join(timeout=2)
         if self.proc is not None:
             self.proc.terminate()
             try:
-                self.out, _ = self.proc.communicate(timeout=5)
+                out, _ = self.proc.communicate(timeout=5)
             except subprocess.TimeoutExpired:
                 self.proc.kill()
-                self.out, _ = self.proc.communicate()
+                out, _ = self.proc.communicate()
+            names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+            bits = {"hw_slowdown": 0x8, "hw_thermal_slowdown": 0x40, "sw_thermal_slowdown": 0x20, "sw_power_cap": 0x4}
+            for r in (out or "").strip().splitlines():
+                c = [x.strip() for x in r.split(",")]
+                if len(c) >= 9 and c[1].isdigit() and c[2].isdigit():
+                    mask = sum(bits[names[k]] for k in range(4) if c[5 + k] == "Active")
+                    self.samples.append((int(c[1]), int(c[2]), mask))
 
     def summary(self):
-        rows = [r.split(",") for r in (self.out or "").strip().splitlines() if r.count(",") >= 8]
-        if not rows:
+        if not self.samples:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
-        sm = [float(r[1]) for r in rows if r[1].strip().replace(".", "").isdigit()]
-        mx = [float(r[2]) for r in rows if r[2].strip().replace(".", "").isdigit()]
-        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
-        reasons = sorted({names[k] for r in rows for k in range(4) if r[5 + k].strip() == "Active"})
-        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
-                "reasons": reasons, "samples": len(rows)}
+        sm = [x[0] for x in self.samples]
+        reasons = sorted({name for x in self.samples for bit, name in self.REASONS.items() if x[2] & bit})
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(x[1] for x in self.samples), "reasons": reasons,
+                "samples": len(self.samples), "source": "nvml" if self.nvml is not None else "nvidia-smi"}
 
 
 # ----------------------------------------------------------------- CPU oracle baseline
@@ -259,31 +314,36 @@ def run_gpu(args):
     stream = torch.cuda.current_stream()
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
 
-    def step(ev=None):
-        if ev is not None:
-            ev[0].record(stream)
+    def step(ev):
+        ev[0].record(stream)
+        mp.plan_and_validate(db, args.policy, buf, stream=stream)
+        ev[1].record(stream)
+
+    def step_separate(ev):
+        ev[0].record(stream)
         mp.live_profile(db, buf.profile, buf.peak_lb, buf.status[0], stream=stream)
-        if ev is not None:
-            ev[1].record(stream)
+        ev[1].record(stream)
         mp.plan_greedy_by_size(db, args.policy, buf.offsets, buf.plan_peak, buf.status[1], workspace=buf.plan_ws,
                                stream=stream)
-        if ev is not None:
-            ev[2].record(stream)
+        ev[2].record(stream)
         mp.validate_plan(db, buf.offsets, buf.verdict, buf.conflict, buf.status[2], workspace=buf.validate_ws,
                          stream=stream)
-        if ev is not None:
-            ev[3].record(stream)
+        ev[3].record(stream)
 
+    mk = lambda k: [torch.cuda.Event(enable_timing=True) for _ in range(k)]
     for _ in range(args.warmup):
         flush.zero_()
-        step()
+        step(mk(2))
+        flush.zero_()
+        step_separate(mk(4))
     torch.cuda.synchronize()
-    st = buf.status.cpu()
-    if not bool((st == 0).all()) or not bool((buf.verdict == 1).all()):
+    step(mk(2))
+    torch.cuda.synchronize()
+    if not bool((buf.status[0] == 0).all()) or not bool((buf.verdict == 1).all()):
         print(json.dumps({"error": "path reported a failed trace or an invalid plan", "rank": rank}))
         return 1
 
-    events = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    events = [mk(2) for _ in range(args.steps)]
     sampler = ClockSampler(gpu_id(dev))
     if dist is not None:
         dist.barrier()
@@ -297,18 +357,19 @@ def run_gpu(args):
         wall = time.perf_counter() - t0
     if dist is not None:
         dist.barrier()
-    per_kernel = [0.0, 0.0, 0.0]
-    step_ms = 0.0
-    for ev in events:
-        for j in range(3):
-            per_kernel[j] += ev[j].elapsed_time(ev[j + 1])
-        step_ms += ev[0].elapsed_time(ev[3])
-    step_ms /= args.steps
-    per_kernel = [x / args.steps for x in per_kernel]
+    step_ms = sum(ev[0].elapsed_time(ev[1]) for ev in events) / args.steps
     step_ms_max = max_over_ranks(step_ms, dist)
     wall_max = max_over_ranks(wall, dist)
     total_tensors = sum_over_ranks(float(ts.n_tensors), dist)
     total_pairs = sum_over_ranks(float(ts.pairs()), dist)
+
+    # The same step as three separate kernels (profile, plan, validate), for the breakdown.
+    sep_events = [mk(4) for _ in range(max(3, args.steps // 2))]
+    for ev in sep_events:
+        flush.zero_()
+        step_separate(ev)
+    torch.cuda.synchronize()
+    per_kernel = [sum(ev[j].elapsed_time(ev[j + 1]) for ev in sep_events) / len(sep_events) for j in range(3)]
 
     # End to end through the host-buffer API: pinned H2D of the inputs, the
     # path, and D2H of every result, each step.
@@ -339,13 +400,14 @@ def run_gpu(args):
     for j, name in enumerate(KERNELS):
         nbytes = algorithmic_bytes(name, ts.n_tensors, ts.n_traces, n_steps)
         gbs = nbytes / (per_kernel[j] * 1e-3) / 1e9
-        kern[name] = {"ms": per_kernel[j], "algorithmic_bytes": nbytes, "achieved_gbs": gbs,
-                      "frac": gbs / peak, "share": per_kernel[j] / sum(per_kernel)}
-    dom = max(KERNELS, key=lambda k: kern[k]["ms"])
-    traffic = ncu_traffic(dom, ts.n_tensors)
-    roof = {"bound": "hbm", "kernel": dom, "achieved": kern[dom]["achieved_gbs"], "peak": peak, "unit": "GB/s",
-            "frac": kern[dom]["frac"], "peak_source": f"{peak_kind} ({'MEASURED_PEAKS.json hbm_gbs' if peak_kind == 'measured' else 'profiling-recipe fallback'})",
-            "traffic": traffic}
+        kern[name] = {"ms": per_kernel[j], "algorithmic_bytes": nbytes, "achieved_gbs": gbs, "frac": gbs / peak}
+    fused_bytes = algorithmic_bytes(FUSED, ts.n_tensors, ts.n_traces, n_steps)
+    fused_gbs = fused_bytes / (step_ms * 1e-3) / 1e9
+    traffic = ncu_traffic(FUSED, ts.n_tensors)
+    roof = {"bound": "hbm", "kernel": "k_plan (fused profile + plan + validate, mp_plan_and_validate)",
+            "achieved": fused_gbs, "peak": peak, "unit": "GB/s", "frac": fused_gbs / peak,
+            "peak_source": f"{peak_kind} ({'MEASURED_PEAKS.json hbm_gbs' if peak_kind == 'measured' else 'profiling-recipe fallback'})",
+            "algorithmic_bytes_per_launch": fused_bytes, "traffic": traffic}
     ob_value, ob_dt, ob_sub = oracle_baseline(ts, args.oracle_traces)
     clocks = sampler.summary()
     line = {
@@ -358,8 +420,9 @@ def run_gpu(args):
                    "parallelism": f"dp{world} (traces sharded by rank, no collective)"},
         "validated_pairs_per_s": total_pairs / (step_ms_max * 1e-3),
         "wall_ms_per_step_incl_flush": 1e3 * wall_max / args.steps,
-        "gpu_launches": 3 * args.steps,
-        "kernels": kern,
+        "gpu_launches": args.steps,
+        "separate_kernels_ms_per_step": sum(per_kernel),
+        "separate_kernels": kern,
         "roofline": roof,
         "cpu_baseline": {"value": ob_value, "unit": UNIT, "cores": 1, "kind": "oracle",
                          "sample": f"first {ob_sub.n_traces} of {ts.n_traces} traces, profile + plan + validate, "

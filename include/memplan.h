@@ -154,6 +154,22 @@ mp_status mp_plan_greedy_by_size(const mp_batch *batch, mp_fit_policy policy, in
 mp_status mp_plan_greedy_by_size_static(const mp_batch *batch, mp_fit_policy policy, int64_t *offsets,
                                         int64_t *plan_peak, int32_t *trace_status, void *stream);
 
+/* The whole path in one pass: each trace is read once and the live profile
+ * (stage 1), the greedy_by_size plan (stage 2) and the validation of that
+ * plan (stage 3) are all computed from it, for batches planned and validated
+ * in one call.  Results are identical to mp_live_profile, then
+ * mp_plan_greedy_by_size, then mp_validate_plan on its offsets; the
+ * validation is a separate pass over the trace in alloc-step order that
+ * checks every lifetime-overlapping pair of the plan just made.
+ * profile / peak_lb: as for mp_live_profile; pass both NULL to skip the
+ * profile (profile_ptr is then not read).  offsets, plan_peak: as for
+ * mp_plan_greedy_by_size.  verdict, conflict (nullable): as for
+ * mp_validate_plan.  One trace_status per trace covers all outputs.
+ * workspace: at least mp_plan_workspace_bytes(batch) bytes. */
+mp_status mp_plan_and_validate(const mp_batch *batch, mp_fit_policy policy, int64_t *profile, int64_t *peak_lb,
+                               int64_t *offsets, int64_t *plan_peak, int32_t *verdict, int32_t *conflict,
+                               int32_t *trace_status, void *workspace, size_t workspace_bytes, void *stream);
+
 /* Bytes of device workspace mp_validate_plan needs for this batch. */
 size_t mp_validate_workspace_bytes(const mp_batch *batch);
 

@@ -9,11 +9,11 @@ include/memplan.h):
 """
 from ._lib import (EINTERNAL, EINVAL, ENOMEM, EOVERFLOW, FIT_BEST, FIT_FIRST, OK, MemplanError,
                    status_string)
-from .api import (DeviceBatch, HostPath, PathBuffers, PathResult, Workspace, live_profile, peak, plan_greedy_by_size,
+from .api import (DeviceBatch, HostPath, PathBuffers, PathResult, Workspace, live_profile, peak, plan_and_validate, plan_greedy_by_size,
                   plan_workspace_bytes, run_path, validate_plan, validate_workspace_bytes)
 
 __all__ = [
-    "DeviceBatch", "HostPath", "PathBuffers", "PathResult", "Workspace", "live_profile", "peak", "plan_greedy_by_size",
+    "DeviceBatch", "HostPath", "PathBuffers", "PathResult", "Workspace", "live_profile", "peak", "plan_and_validate", "plan_greedy_by_size",
     "plan_workspace_bytes", "run_path", "validate_plan", "validate_workspace_bytes", "MemplanError",
     "status_string", "OK", "EINVAL", "EOVERFLOW", "ENOMEM", "EINTERNAL", "FIT_FIRST", "FIT_BEST",
 ]

@@ -19,6 +19,7 @@ EXPORTS = (
     "mp_plan_workspace_bytes",
     "mp_plan_greedy_by_size",
     "mp_plan_greedy_by_size_static",
+    "mp_plan_and_validate",
     "mp_validate_workspace_bytes",
     "mp_validate_plan",
     "mp_peak",
@@ -74,6 +75,8 @@ def load(path: str = LIB_PATH):
     lib.mp_plan_greedy_by_size.restype = i32
     lib.mp_plan_greedy_by_size_static.argtypes = [BP, i32, P, P, P, P]
     lib.mp_plan_greedy_by_size_static.restype = i32
+    lib.mp_plan_and_validate.argtypes = [BP, i32, P, P, P, P, P, P, P, P, sz, P]
+    lib.mp_plan_and_validate.restype = i32
     lib.mp_validate_workspace_bytes.argtypes = [BP]
     lib.mp_validate_workspace_bytes.restype = sz
     lib.mp_validate_plan.argtypes = [BP, P, P, P, P, P, sz, P]

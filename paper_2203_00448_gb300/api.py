@@ -184,6 +184,27 @@ def validate_plan(batch: DeviceBatch, offsets: torch.Tensor, verdict=None, confl
     return verdict, (conflict.view(-1, 2) if conflict is not None else None), status
 
 
+def plan_and_validate(batch: DeviceBatch, policy="first", buffers: "PathBuffers | None" = None, profile: bool = True,
+                      stream=None) -> "PathResult":
+    """The whole path in one kernel pass: profile (optional), greedy_by_size plan and its validation.
+
+    Same results as live_profile + plan_greedy_by_size + validate_plan; the
+    single status row applies to every output of a trace.
+    """
+    lib = _lib.load()
+    buf = buffers or PathBuffers(batch)
+    s = batch.struct()
+    need = int(lib.mp_plan_workspace_bytes(ctypes.byref(s)))
+    wptr, wbytes = buf.plan_ws.get(need)
+    _check("mp_plan_and_validate",
+           lib.mp_plan_and_validate(ctypes.byref(s), _policy(policy), _ptr(buf.profile) if profile else None,
+                                    _ptr(buf.peak_lb) if profile else None, _ptr(buf.offsets), _ptr(buf.plan_peak),
+                                    _ptr(buf.verdict), _ptr(buf.conflict), _ptr(buf.status[0]), wptr, wbytes,
+                                    _stream_ptr(stream)))
+    return PathResult(buf.profile, buf.peak_lb, buf.offsets, buf.plan_peak, buf.verdict,
+                      buf.conflict.view(-1, 2), buf.status[0])
+
+
 def peak(batch: DeviceBatch, offsets: torch.Tensor, plan_peak=None, status=None, stream=None):
     """total_mem of a given plan per trace: max(offset + size)."""
     lib, dev = _lib.load(), batch.device
@@ -239,7 +260,8 @@ def run_path(batch: DeviceBatch, policy="first", buffers: PathBuffers | None = N
 
 class HostPath:
     """End-to-end use from host memory: copies a batch from pinned host buffers
-    to the device, runs the whole path, and copies every result back.
+    to the device, runs the whole path (one plan_and_validate call), and copies
+    every result back.
 
     ``run(ts)`` takes a host batch (numpy arrays, e.g. tracegen.TraceSet) with
     the same shape as the one the object was built for and returns host
@@ -257,8 +279,9 @@ class HostPath:
         self.host_in = {k: torch.empty(tuple(getattr(self.dev_batch, k).shape), dtype=getattr(self.dev_batch, k).dtype,
                                        pin_memory=True) for k in self._IN}
         self._outs = ("profile", "peak_lb", "offsets", "plan_peak", "verdict", "conflict", "status")
-        self.host_out = {k: torch.empty(tuple(getattr(self.buffers, k).shape), dtype=getattr(self.buffers, k).dtype,
-                                        pin_memory=True) for k in self._outs}
+        shape = lambda k: tuple(getattr(self.buffers, k).shape[1:] if k == "status" else getattr(self.buffers, k).shape)
+        self.host_out = {k: torch.empty(shape(k), dtype=getattr(self.buffers, k).dtype, pin_memory=True)
+                         for k in self._outs}
 
     @property
     def h2d_bytes(self) -> int:
@@ -280,8 +303,9 @@ class HostPath:
         with torch.cuda.stream(s):
             for k in self._IN:
                 getattr(self.dev_batch, k).copy_(self.host_in[k], non_blocking=True)
-            run_path(self.dev_batch, self.policy, self.buffers, stream=s)
+            plan_and_validate(self.dev_batch, self.policy, self.buffers, stream=s)
             for k in self._outs:
-                self.host_out[k].copy_(getattr(self.buffers, k), non_blocking=True)
+                src = getattr(self.buffers, k)
+                self.host_out[k].copy_(src[0] if k == "status" else src, non_blocking=True)
         s.synchronize()
         return {k: v.numpy() for k, v in self.host_out.items()}

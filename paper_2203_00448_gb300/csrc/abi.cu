@@ -117,6 +117,28 @@ __attribute__((visibility("default"))) mp_status mp_plan_greedy_by_size(
                                      static_cast<cudaStream_t>(stream)));
 }
 
+__attribute__((visibility("default"))) mp_status mp_plan_and_validate(
+    const mp_batch* batch, mp_fit_policy policy, int64_t* profile, int64_t* peak_lb, int64_t* offsets,
+    int64_t* plan_peak, int32_t* verdict, int32_t* conflict, int32_t* trace_status, void* workspace,
+    size_t workspace_bytes, void* stream) {
+    const bool want_profile = profile != nullptr || peak_lb != nullptr;
+    mp_status st = check_batch(batch, want_profile);
+    if (st != MP_OK) return st;
+    if (policy != MP_FIT_FIRST && policy != MP_FIT_BEST) return MP_EINVAL;
+    if (batch->max_tensors > mp::kPlanMaxTensors) return MP_EINVAL;
+    if (want_profile && (!array_ok(profile, batch->n_steps) || !array_ok(peak_lb, batch->n_traces)))
+        return MP_EINVAL;
+    if (!array_ok(offsets, batch->n_tensors) || !array_ok(plan_peak, batch->n_traces) ||
+        !array_ok(verdict, batch->n_traces) || !array_ok(trace_status, batch->n_traces))
+        return MP_EINVAL;
+    if (conflict != nullptr && !aligned(conflict)) return MP_EINVAL;
+    st = check_workspace(mp::plan_workspace_bytes(*batch), workspace, workspace_bytes);
+    if (st != MP_OK) return st;
+    return from_cuda(mp::launch_plan_fused(*batch, (int32_t)policy, want_profile ? profile : nullptr,
+                                           want_profile ? peak_lb : nullptr, offsets, plan_peak, verdict, conflict,
+                                           trace_status, workspace, static_cast<cudaStream_t>(stream)));
+}
+
 __attribute__((visibility("default"))) size_t mp_validate_workspace_bytes(const mp_batch* batch) {
     if (check_batch(batch, false) != MP_OK) return 0;
     return mp::validate_workspace_bytes(*batch);

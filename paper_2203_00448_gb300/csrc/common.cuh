@@ -71,6 +71,16 @@ __device__ __forceinline__ void atomic_add_u64_split(int64_t* word, uint64_t v) 
     if (h) atomicAdd(w + 1, h);
 }
 
+// Difference arrays of the live profile are scanned kProfRun consecutive steps
+// per lane; in shared memory each run is followed by kProfPad int64 of padding
+// so that the lanes' 16-byte reads of their runs fall in distinct banks.
+constexpr int kProfRun = 16;
+constexpr int kProfPad = 2;
+__host__ __device__ constexpr int64_t prof_pos(int64_t t) { return t + kProfPad * (t / kProfRun); }
+__host__ __device__ constexpr size_t prof_padded(size_t T) {
+    return T + kProfPad * ((T + kProfRun - 1) / kProfRun);
+}
+
 // ------------------------------------------------------------ warp level
 
 __device__ __forceinline__ uint64_t warp_sat_sum(uint64_t v) {

@@ -46,5 +46,8 @@ constexpr int32_t kPlanMaxTensors = (1 << 28) - 1;
 size_t plan_workspace_bytes(const mp_batch& bt);
 cudaError_t launch_plan(const mp_batch& bt, int32_t policy, int64_t* offsets, int64_t* plan_peak,
                         int32_t* status, void* workspace, cudaStream_t stream);
+cudaError_t launch_plan_fused(const mp_batch& bt, int32_t policy, int64_t* profile, int64_t* peak_lb,
+                              int64_t* offsets, int64_t* plan_peak, int32_t* verdict, int32_t* conflict,
+                              int32_t* status, void* workspace, cudaStream_t stream);
 
 }  // namespace mp

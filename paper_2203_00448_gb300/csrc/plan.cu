@@ -73,16 +73,30 @@ struct SRec {
 
 template <typename I>
 struct PlanLayout {
-    size_t arec, offid, bend, cst, lst, xl, total;
-    __host__ __device__ PlanLayout(int64_t n, int64_t T) {
+    size_t arec, offid, bend, cst, lst, xl, dprof, total;
+    __host__ __device__ PlanLayout(int64_t n, int64_t T, bool fused) {
         arec = 0;
         offid = arec + align16((size_t)n * sizeof(ARec<I>));
         bend = offid + align16((size_t)n * 8);
         cst = bend + align16((size_t)T * 4);
         lst = cst + align16((size_t)(n + 1) * 4);
         xl = lst + align16((size_t)n * sizeof(I));
-        total = align_up(xl + align16((size_t)n * sizeof(I)));
+        dprof = xl + align16((size_t)n * sizeof(I));
+        total = align_up(dprof + (fused ? align16(prof_padded((size_t)T) * 8) : 0));
     }
+};
+
+// Outputs of one launch; the fused kernel also fills the profile, its peak,
+// the verdict and the conflict pair (the last three pointers may be null).
+struct PlanOut {
+    int32_t policy;
+    int64_t* offsets;
+    int64_t* plan_peak;
+    int32_t* status;
+    int64_t* profile;
+    int64_t* peak_lb;
+    int32_t* verdict;
+    int32_t* conflict;
 };
 
 // x strictly precedes y in priority (size desc, alloc asc, id asc).
@@ -433,23 +447,25 @@ __device__ void place_large(SRec<I>* R, int32_t c, int32_t policy, int64_t* bo, 
     }
 }
 
-template <typename I, bool kSmem>
+template <typename I, bool kSmem, bool kFused>
 __global__ void __launch_bounds__(kSmem ? kPlanThreadsSmem : kPlanThreadsGlobal)
-k_plan(mp_batch bt, int32_t policy, int64_t* __restrict__ offsets, int64_t* __restrict__ plan_peak,
-       int32_t* __restrict__ status, unsigned char* __restrict__ ws, size_t data_stride, size_t buf_offset,
+k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_stride, size_t buf_offset,
        size_t buf_stride) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     __shared__ int64_t red[72];
     __shared__ int32_t s_cnt, s_nt, s_nw, s_nx, s_bad;
-    __shared__ unsigned long long s_top, s_hi, s_lo, s_max;
+    __shared__ unsigned long long s_top, s_hi, s_lo, s_max, s_key, s_lbmax;
     const int b = blockIdx.x;
-    const TraceView tv = load_trace(bt, b, false);
+    const int32_t policy = out.policy;
+    int32_t* __restrict__ status = out.status;
+    const bool want_profile = kFused && out.profile != nullptr;
+    const TraceView tv = load_trace(bt, b, want_profile);
     if (tv.st != MP_OK) {
         if (threadIdx.x == 0) status[b] = tv.st;
         return;
     }
     const int32_t n = tv.n, T = tv.T;
-    const PlanLayout<I> L(kSmem ? n : bt.max_tensors, kSmem ? T : bt.max_steps);
+    const PlanLayout<I> L(kSmem ? n : bt.max_tensors, kSmem ? T : bt.max_steps, kFused);
     unsigned char* base = kSmem ? smem_raw : ws + (size_t)b * data_stride;
     ARec<I>* AR = reinterpret_cast<ARec<I>*>(base + L.arec);
     int64_t* OFFID = reinterpret_cast<int64_t*>(base + L.offid);
@@ -468,7 +484,8 @@ k_plan(mp_batch bt, int32_t policy, int64_t* __restrict__ offsets, int64_t* __re
     if (threadIdx.x == 0) {
         s_nt = s_nw = s_nx = 0;
         s_bad = 0;
-        s_hi = s_lo = s_max = 0;
+        s_hi = s_lo = s_max = s_lbmax = 0;
+        s_key = ~0ull;
     }
     __syncthreads();
     const int32_t* __restrict__ Ag = bt.alloc_step + tv.lo;
@@ -505,7 +522,11 @@ k_plan(mp_batch bt, int32_t policy, int64_t* __restrict__ offsets, int64_t* __re
     if (!ok) s_bad = 1;
     __syncthreads();
     if (s_bad || size_sum_overflows(s_hi, s_lo)) {
-        if (threadIdx.x == 0) status[b] = s_bad ? MP_EINVAL : MP_EOVERFLOW;
+        if (threadIdx.x == 0) {
+            status[b] = s_bad ? MP_EINVAL : MP_EOVERFLOW;
+            if (kFused && out.verdict) out.verdict[b] = 0;
+            if (kFused && out.conflict) out.conflict[2 * b] = out.conflict[2 * b + 1] = -1;
+        }
         return;
     }
 
@@ -522,6 +543,60 @@ k_plan(mp_batch bt, int32_t policy, int64_t* __restrict__ offsets, int64_t* __re
         AR[atomicAdd(BEND + a, 1)] = r;
     }
     __syncthreads();
+
+    // ---- live profile from the records (fused): difference array, scan, write
+    if (want_profile) {
+        int64_t* D = reinterpret_cast<int64_t*>(base + L.dprof);
+        const int64_t dlen = (int64_t)prof_padded((size_t)T);
+        for (int64_t t = threadIdx.x; t < dlen; t += blockDim.x) D[t] = 0;
+        __syncthreads();
+        for (int p = threadIdx.x; p < n; p += blockDim.x) {
+            const ARec<I> r = AR[p];
+            atomic_add_u64_split(D + prof_pos(r.a), (uint64_t)r.s);
+            if (r.f < T) atomic_add_u64_split(D + prof_pos(r.f), (uint64_t)(-r.s));
+        }
+        __syncthreads();
+        int64_t* pout = out.profile + tv.plo;
+        const bool vec_out = (reinterpret_cast<uintptr_t>(pout) & 15) == 0;
+        int64_t carry = 0, lmax = 0;
+        for (int64_t base_t = 0; base_t < T; base_t += (int64_t)blockDim.x * kProfRun) {
+            const int64_t my = base_t + (int64_t)threadIdx.x * kProfRun;
+            const int64_t* run = D + prof_pos(my);
+            int64_t v[kProfRun];
+#pragma unroll
+            for (int k = 0; k < kProfRun; k += 2) {
+                if (my + kProfRun <= T) {
+                    const longlong2 q = *reinterpret_cast<const longlong2*>(run + k);
+                    v[k] = q.x;
+                    v[k + 1] = q.y;
+                } else {
+                    v[k] = my + k < T ? run[k] : 0;
+                    v[k + 1] = my + k + 1 < T ? run[k + 1] : 0;
+                }
+            }
+#pragma unroll
+            for (int k = 1; k < kProfRun; ++k) v[k] += v[k - 1];
+            int64_t tot;
+            const int64_t pre = block_excl_scan<int64_t>(v[kProfRun - 1], red, &tot) + carry;
+#pragma unroll
+            for (int k = 0; k < kProfRun; ++k) {
+                v[k] += pre;
+                lmax = v[k] > lmax ? v[k] : lmax;
+            }
+            if (vec_out && my + kProfRun <= T) {
+#pragma unroll
+                for (int k = 0; k < kProfRun; k += 2)
+                    *reinterpret_cast<longlong2*>(pout + my + k) = make_longlong2(v[k], v[k + 1]);
+            } else {
+#pragma unroll
+                for (int k = 0; k < kProfRun; ++k)
+                    if (my + k < T) pout[my + k] = v[k];
+            }
+            carry += tot;
+        }
+        lmax = warp_max_i64(lmax);
+        if ((threadIdx.x & 31) == 0 && lmax > 0) atomicMax(&s_lbmax, (unsigned long long)lmax);
+    }
 
     // ---- components: a run starts where no earlier tensor is live any more
     const int32_t chunk = (n + blockDim.x - 1) / blockDim.x;
@@ -608,13 +683,45 @@ k_plan(mp_batch bt, int32_t policy, int64_t* __restrict__ offsets, int64_t* __re
         __syncthreads();
     }
 
-    // ---- offsets out, plan peak
     mx = warp_max_i64(mx);
     if ((threadIdx.x & 31) == 0 && mx > 0) atomicMax(&s_max, (unsigned long long)mx);
     __syncthreads();
-    for (int k = threadIdx.x; k < n; k += blockDim.x) offsets[tv.lo + k] = OFFID[k];
+
+    // ---- validation of the plan just made (fused): every lifetime-overlapping
+    // pair once, from its earlier member in alloc order, is checked for address
+    // overlap -- an independent pass over the alloc-ordered records
+    if (kFused) {
+        for (int p = threadIdx.x; p < n; p += blockDim.x) {
+            const ARec<I> ri = AR[p];
+            const int32_t stop = BEND[ri.f - 1];  // tensors with alloc < free_i
+            if (stop <= p + 1) continue;
+            const int64_t oi = OFFID[ri.id], ei = oi + ri.s;
+            for (int q = p + 1; q < stop; ++q) {
+                const ARec<I> rj = AR[q];
+                const int64_t oj = OFFID[rj.id];
+                if (oi < oj + rj.s && oj < ei) {
+                    const uint32_t i = (uint32_t)ri.id, j = (uint32_t)rj.id;
+                    atomicMin(&s_key, ((unsigned long long)(i < j ? i : j) << 32) | (i < j ? j : i));
+                }
+            }
+        }
+        __syncthreads();
+    }
+
+    // ---- outputs
+    for (int k = threadIdx.x; k < n; k += blockDim.x) out.offsets[tv.lo + k] = OFFID[k];
     if (threadIdx.x == 0) {
-        plan_peak[b] = (int64_t)s_max;
+        out.plan_peak[b] = (int64_t)s_max;
+        if (kFused) {
+            if (want_profile && out.peak_lb) out.peak_lb[b] = (int64_t)s_lbmax;
+            const unsigned long long key = s_key;
+            const bool ok = key == ~0ull;
+            if (out.verdict) out.verdict[b] = ok ? 1 : 0;
+            if (out.conflict) {
+                out.conflict[2 * b] = ok ? -1 : (int32_t)(key >> 32);
+                out.conflict[2 * b + 1] = ok ? -1 : (int32_t)(key & 0xffffffffu);
+            }
+        }
         status[b] = MP_OK;
     }
 }
@@ -629,11 +736,11 @@ struct PlanGeometry {
 // workspace always holds the CTA tier's buffers (predecessor offsets / ends,
 // the index list of a large component, and its records in priority order),
 // sized for up to max_tensors.
-PlanGeometry plan_geometry(const mp_batch& bt) {
+PlanGeometry plan_geometry(const mp_batch& bt, bool fused) {
     PlanGeometry g;
     g.narrow = bt.max_tensors < 32767 && bt.max_steps <= 32767;
-    g.data = g.narrow ? PlanLayout<int16_t>(bt.max_tensors, bt.max_steps).total
-                      : PlanLayout<int32_t>(bt.max_tensors, bt.max_steps).total;
+    g.data = g.narrow ? PlanLayout<int16_t>(bt.max_tensors, bt.max_steps, fused).total
+                      : PlanLayout<int32_t>(bt.max_tensors, bt.max_steps, fused).total;
     g.smem = g.data <= kPlanSmemLimit;
     g.data_stride = g.smem ? 0 : g.data;
     g.buf_offset = (size_t)bt.n_traces * g.data_stride;
@@ -643,33 +750,51 @@ PlanGeometry plan_geometry(const mp_batch& bt) {
     return g;
 }
 
-template <typename I, bool kSmem>
-cudaError_t launch_variant(const mp_batch& bt, const PlanGeometry& g, int32_t policy, int64_t* offsets,
-                           int64_t* plan_peak, int32_t* status, unsigned char* ws, cudaStream_t stream) {
+template <typename I, bool kSmem, bool kFused>
+cudaError_t launch_variant(const mp_batch& bt, const PlanGeometry& g, const PlanOut& out, unsigned char* ws,
+                           cudaStream_t stream) {
     const size_t smem = kSmem ? g.data : 0;
     if (kSmem) {
-        cudaError_t e = set_smem_limit((const void*)k_plan<I, kSmem>, smem);
+        cudaError_t e = set_smem_limit((const void*)k_plan<I, kSmem, kFused>, smem);
         if (e != cudaSuccess) return e;
     }
-    k_plan<I, kSmem><<<(unsigned)bt.n_traces, kSmem ? kPlanThreadsSmem : kPlanThreadsGlobal, smem, stream>>>(
-        bt, policy, offsets, plan_peak, status, ws, g.data_stride, g.buf_offset, g.buf_stride);
+    k_plan<I, kSmem, kFused>
+        <<<(unsigned)bt.n_traces, kSmem ? kPlanThreadsSmem : kPlanThreadsGlobal, smem, stream>>>(
+            bt, out, ws, g.data_stride, g.buf_offset, g.buf_stride);
     return cudaGetLastError();
+}
+
+template <bool kFused>
+cudaError_t launch_any(const mp_batch& bt, const PlanOut& out, void* workspace, cudaStream_t stream) {
+    if (bt.n_traces == 0) return cudaSuccess;
+    const PlanGeometry g = plan_geometry(bt, kFused);
+    unsigned char* ws = static_cast<unsigned char*>(workspace);
+    if (g.narrow)
+        return g.smem ? launch_variant<int16_t, true, kFused>(bt, g, out, ws, stream)
+                      : launch_variant<int16_t, false, kFused>(bt, g, out, ws, stream);
+    return g.smem ? launch_variant<int32_t, true, kFused>(bt, g, out, ws, stream)
+                  : launch_variant<int32_t, false, kFused>(bt, g, out, ws, stream);
 }
 
 }  // namespace
 
-size_t plan_workspace_bytes(const mp_batch& bt) { return plan_geometry(bt).workspace; }
+// One workspace size serves both the planner and the fused entry point.
+size_t plan_workspace_bytes(const mp_batch& bt) {
+    const size_t a = plan_geometry(bt, false).workspace, b = plan_geometry(bt, true).workspace;
+    return a > b ? a : b;
+}
 
 cudaError_t launch_plan(const mp_batch& bt, int32_t policy, int64_t* offsets, int64_t* plan_peak,
                         int32_t* status, void* workspace, cudaStream_t stream) {
-    if (bt.n_traces == 0) return cudaSuccess;
-    const PlanGeometry g = plan_geometry(bt);
-    unsigned char* ws = static_cast<unsigned char*>(workspace);
-    if (g.narrow)
-        return g.smem ? launch_variant<int16_t, true>(bt, g, policy, offsets, plan_peak, status, ws, stream)
-                      : launch_variant<int16_t, false>(bt, g, policy, offsets, plan_peak, status, ws, stream);
-    return g.smem ? launch_variant<int32_t, true>(bt, g, policy, offsets, plan_peak, status, ws, stream)
-                  : launch_variant<int32_t, false>(bt, g, policy, offsets, plan_peak, status, ws, stream);
+    const PlanOut out{policy, offsets, plan_peak, status, nullptr, nullptr, nullptr, nullptr};
+    return launch_any<false>(bt, out, workspace, stream);
+}
+
+cudaError_t launch_plan_fused(const mp_batch& bt, int32_t policy, int64_t* profile, int64_t* peak_lb,
+                              int64_t* offsets, int64_t* plan_peak, int32_t* verdict, int32_t* conflict,
+                              int32_t* status, void* workspace, cudaStream_t stream) {
+    const PlanOut out{policy, offsets, plan_peak, status, profile, peak_lb, verdict, conflict};
+    return launch_any<true>(bt, out, workspace, stream);
 }
 
 }  // namespace mp

@@ -25,18 +25,15 @@ namespace mp {
 
 namespace {
 
-constexpr int kScanItems = 16;  // profile steps per lane per tile (a power of two)
-constexpr int kPad = 2;         // int64 padding after every kScanItems entries in shared memory
+constexpr int kScanItems = kProfRun;  // profile steps per lane per tile
 
 // Position of step t in the (padded, when kSmem) difference array.
 template <bool kSmem>
 __device__ __forceinline__ int64_t dpos(int64_t t) {
-    return kSmem ? t + kPad * (t / kScanItems) : t;
+    return kSmem ? prof_pos(t) : t;
 }
 
-__host__ __device__ constexpr size_t padded_steps(size_t T) {
-    return T + kPad * ((T + kScanItems - 1) / kScanItems);
-}
+__host__ __device__ constexpr size_t padded_steps(size_t T) { return prof_padded(T); }
 
 // Adds one tensor to the difference array; returns false if it is invalid.
 template <bool kSmem>

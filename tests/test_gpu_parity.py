@@ -222,3 +222,53 @@ def test_generator_and_oracle_stable_on_this_host(cuda_lib):
         o = config_oracle(k, oracle.FIT_FIRST)
         assert int(o["offsets"].sum()) == c["first_offsets_sum"]
         assert int(o["plan_peak"].sum()) == c["first_plan_peak_sum"]
+
+
+# ------------------------------------------------------------- fused entry point
+
+def fused_run(ts, policy, profile=True):
+    import paper_2203_00448_gb300 as mp
+
+    db = mp.DeviceBatch.from_host(ts, "cuda")
+    res = mp.plan_and_validate(db, policy, profile=profile)
+    torch.cuda.synchronize()
+    h = lambda t: t.cpu().numpy()
+    return dict(profile=h(res.profile), peak_lb=h(res.peak_lb), offsets=h(res.offsets), plan_peak=h(res.plan_peak),
+                verdict=h(res.verdict), conflict=h(res.conflict), st=h(res.status))
+
+
+def assert_fused_parity(ts, g, o, profile=True):
+    st_expect = o["st"].max(axis=0)  # a trace's one status: its error, if any stage reports one
+    assert np.array_equal(g["st"], st_expect), "trace status differs"
+    ok = st_expect == 0
+    for b in np.nonzero(ok)[0]:
+        lo, hi = ts.trace_ptr[b], ts.trace_ptr[b + 1]
+        assert np.array_equal(g["offsets"][lo:hi], o["offsets"][lo:hi]), f"offsets of trace {b}"
+        if profile:
+            plo, phi = ts.profile_ptr[b], ts.profile_ptr[b + 1]
+            assert np.array_equal(g["profile"][plo:phi], o["profile"][plo:phi]), f"profile of trace {b}"
+    for k in ("plan_peak", "verdict") + (("peak_lb",) if profile else ()):
+        assert np.array_equal(g[k][ok], o[k][ok]), k
+    assert np.array_equal(g["conflict"][ok], o["conflict"][ok])
+    assert (g["verdict"][ok] == 1).all()
+
+
+@pytest.mark.parametrize("name,pol", POLICIES)
+@pytest.mark.parametrize("k", range(5))
+def test_fused_workload_parity(cuda_lib, k, name, pol):
+    ts = tg.config(k)
+    assert_fused_parity(ts, fused_run(ts, name), config_oracle(k, pol))
+
+
+@pytest.mark.parametrize("name,pol", POLICIES)
+def test_fused_random_and_errors(cuda_lib, name, pol):
+    for ts in (tg.random_small(11, 300, 120, 200, 1 << 20), tg.random_small(12, 100, 300, 2000, 1 << 30),
+               tg.from_tuples([(4, [(-1, 2, 8)]), (4, [(0, 1, 2 ** 62), (0, 2, 2 ** 62)]), (0, []), (5, []),
+                               (6, [(0, 3, 64), (1, 4, 32), (3, 6, 8)])])):
+        assert_fused_parity(ts, fused_run(ts, name), oracle_run(ts, pol))
+
+
+def test_fused_without_profile(cuda_lib):
+    ts = tg.config(2).select(range(0, 4096, 16))
+    o = oracle_run(ts, oracle.FIT_FIRST)
+    assert_fused_parity(ts, fused_run(ts, "first", profile=False), o, profile=False)
