@@ -306,8 +306,9 @@ def run_gpu(args):
 
     build.build()
     w = WORKLOAD
-    ts = tracegen.random_batch(shard_seed0(rank), w["n_traces"], w["n"], w["T"], w["p"], w["lo_e"], w["hi_e"],
-                               name=WORKLOAD_NAME)
+    ts = tracegen.random_batch(shard_seed0(rank, args.traces), args.traces, w["n"], w["T"], w["p"], w["lo_e"],
+                               w["hi_e"], name=WORKLOAD_NAME if args.traces == w["n_traces"] else
+                               f"batched-random-{args.traces}x512x1024")
     dev = torch.device("cuda", torch.cuda.current_device())
     db = mp.DeviceBatch.from_host(ts, dev)
     buf = mp.PathBuffers(db)
@@ -334,8 +335,9 @@ def run_gpu(args):
     for _ in range(args.warmup):
         flush.zero_()
         step(mk(2))
-        flush.zero_()
-        step_separate(mk(4))
+        if not args.no_breakdown:
+            flush.zero_()
+            step_separate(mk(4))
     torch.cuda.synchronize()
     step(mk(2))
     torch.cuda.synchronize()
@@ -364,12 +366,14 @@ def run_gpu(args):
     total_pairs = sum_over_ranks(float(ts.pairs()), dist)
 
     # The same step as three separate kernels (profile, plan, validate), for the breakdown.
-    sep_events = [mk(4) for _ in range(max(3, args.steps // 2))]
-    for ev in sep_events:
-        flush.zero_()
-        step_separate(ev)
-    torch.cuda.synchronize()
-    per_kernel = [sum(ev[j].elapsed_time(ev[j + 1]) for ev in sep_events) / len(sep_events) for j in range(3)]
+    per_kernel = [float("nan")] * 3
+    if not args.no_breakdown:
+        sep_events = [mk(4) for _ in range(max(3, args.steps // 2))]
+        for ev in sep_events:
+            flush.zero_()
+            step_separate(ev)
+        torch.cuda.synchronize()
+        per_kernel = [sum(ev[j].elapsed_time(ev[j + 1]) for ev in sep_events) / len(sep_events) for j in range(3)]
 
     # End to end through the host-buffer API: pinned H2D of the inputs, the
     # path, and D2H of every result, each step.
@@ -396,8 +400,8 @@ def run_gpu(args):
         return 0
     peak, peak_kind = measured_peaks()
     n_steps = ts.n_steps
-    kern = {}
-    for j, name in enumerate(KERNELS):
+    kern = None if args.no_breakdown else {}
+    for j, name in enumerate(KERNELS if not args.no_breakdown else ()):
         nbytes = algorithmic_bytes(name, ts.n_tensors, ts.n_traces, n_steps)
         gbs = nbytes / (per_kernel[j] * 1e-3) / 1e9
         kern[name] = {"ms": per_kernel[j], "algorithmic_bytes": nbytes, "achieved_gbs": gbs, "frac": gbs / peak}
@@ -408,7 +412,13 @@ def run_gpu(args):
             "achieved": fused_gbs, "peak": peak, "unit": "GB/s", "frac": fused_gbs / peak,
             "peak_source": f"{peak_kind} ({'MEASURED_PEAKS.json hbm_gbs' if peak_kind == 'measured' else 'profiling-recipe fallback'})",
             "algorithmic_bytes_per_launch": fused_bytes, "traffic": traffic}
-    ob_value, ob_dt, ob_sub = oracle_baseline(ts, args.oracle_traces)
+    if args.oracle_traces > 0:
+        ob_value, ob_dt, ob_sub = oracle_baseline(ts, args.oracle_traces)
+        cpu_baseline = {"value": ob_value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                        "sample": f"first {ob_sub.n_traces} of {ts.n_traces} traces, profile + plan + validate, "
+                                  f"{ob_dt:.2f} s single-threaded"}
+    else:
+        cpu_baseline = None
     clocks = sampler.summary()
     line = {
         "metric": METRIC, "value": total_tensors / (step_ms_max * 1e-3), "unit": UNIT, "n_gpus": world,
@@ -421,12 +431,10 @@ def run_gpu(args):
         "validated_pairs_per_s": total_pairs / (step_ms_max * 1e-3),
         "wall_ms_per_step_incl_flush": 1e3 * wall_max / args.steps,
         "gpu_launches": args.steps,
-        "separate_kernels_ms_per_step": sum(per_kernel),
+        "separate_kernels_ms_per_step": None if args.no_breakdown else sum(per_kernel),
         "separate_kernels": kern,
         "roofline": roof,
-        "cpu_baseline": {"value": ob_value, "unit": UNIT, "cores": 1, "kind": "oracle",
-                         "sample": f"first {ob_sub.n_traces} of {ts.n_traces} traces, profile + plan + validate, "
-                                   f"{ob_dt:.2f} s single-threaded"},
+        "cpu_baseline": cpu_baseline,
         "e2e": e2e,
         "clocks": clocks,
     }
@@ -446,6 +454,10 @@ def main(argv=None):
     ap.add_argument("--oracle-traces", type=int, default=4096,
                     help="traces of the workload the CPU-baseline leg runs through the oracle")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-breakdown", action="store_true",
+                    help="skip the three-kernel breakdown (profiling runs that should launch the fused kernel only)")
+    ap.add_argument("--traces", type=int, default=WORKLOAD["n_traces"],
+                    help="traces per rank (the reported workload is the default 4096; other values are for profiling)")
     args = ap.parse_args(argv)
     if args.impl == "reference":
         return run_reference(args)
