@@ -1,5 +1,6 @@
 // plan.cu -- stage 2: greedy_by_size offset assignment (Sec. 2.3; the default
-// strategy of Sec. 3.2).
+// strategy of Sec. 3.2), and the fused pass that also builds the live profile
+// (stage 1) and validates the plan (stage 3).
 //
 // Definition (sequential): take tensors in priority order -- size descending,
 // alloc step ascending, id ascending -- and give each, among the already
@@ -14,18 +15,20 @@
 // earlier tensor is still live at alloc(p) (the running maximum of free steps
 // is <= alloc(p)).  Each component is then placed by the sequential
 // definition itself:
-//   - at most kThreadComp tensors: one thread, entirely in registers (a
-//     sorting network into priority order, then placement one by one);
+//   - one tensor: offset 0;
+//   - at most kThreadComp tensors: one thread.  First, one thread per tensor
+//     finds its priority rank inside its component and the mask of members
+//     that both precede it and overlap its lifetime (inside an alloc-ordered
+//     run, j < i overlaps i iff f_j > a_i, and j > i iff a_j < f_i); then one
+//     thread per component visits the members in rank order;
 //   - at most kWarpComp tensors: one warp, a tensor per lane; each lane counts
-//     the members that precede it (its priority rank), then the warp places
-//     rank 0, 1, ... in turn, every placed lane testing its own tensor as a
-//     predecessor, with single-instruction warp reductions;
+//     the members that precede it, then the warp places rank 0, 1, ... in
+//     turn with single-instruction warp reductions;
 //   - larger: the whole CTA bitonic-sorts the component into priority order,
 //     then places it tensor by tensor with a CTA-wide gather of the
 //     overlapping placed tensors and a CTA-wide gap search.
-// Batches of short-lived traces split into hundreds of tiny components per
-// trace, so nearly all work runs thread- or warp-parallel with no per-tensor
-// barrier.
+// Thread-tier components are handed out largest size class first, so the
+// lanes of a warp carry similar work.
 //
 // Gap search.  FIRST is the lowest offset o at which [o, o + s_i) meets no
 // predecessor [off_j, end_j).  One thread: start at o = 0 and jump to the
@@ -39,6 +42,12 @@
 // by min{off_j >= c} - c).  CTA, many predecessors: FIRST by the jump method
 // with block reductions; BEST by sorting the predecessors by offset and
 // scanning the running maximum end, which exposes every gap at once.
+//
+// Fused pass (mp_plan_and_validate): the difference array of the profile is
+// built while the inputs are first read, scanned and written out before the
+// records are scattered over the same shared memory; after placement every
+// lifetime-overlapping pair is checked once, from its earlier member in alloc
+// order, for address overlap.
 #include "common.cuh"
 #include "launch.h"
 
@@ -46,10 +55,18 @@ namespace mp {
 
 namespace {
 
-constexpr int32_t kThreadComp = 4;  // components up to this size: one thread (registers)
-constexpr int32_t kWarpComp = 32;   // ... up to this size: one warp (a tensor per lane); else the CTA
-constexpr int32_t kCandMax = 64;    // CTA tier: up to this many predecessors, test all candidates
+constexpr int32_t kThreadComp = 8;   // components up to this size: one thread
+constexpr int32_t kWarpComp = 32;    // ... up to this size: one warp (a tensor per lane); else the CTA
+constexpr int32_t kCandMax = 64;     // CTA tier: up to this many predecessors, test all candidates
+constexpr int kCached = 4;           // tensors per thread kept in registers between the two input passes
 constexpr int64_t kNone = INT64_MAX;
+
+// Component size classes for the counting sort of the component list:
+// classes 0 .. kThreadComp - 2 hold sizes kThreadComp down to 2 (thread tier,
+// largest first), then one class for the warp tier and one for the CTA tier.
+constexpr int kBinWarp = kThreadComp - 1;
+constexpr int kBinCta = kThreadComp;
+constexpr int kBins = kThreadComp + 1;
 
 __host__ __device__ constexpr size_t align16(size_t x) { return (x + 15) & ~size_t(15); }
 
@@ -59,7 +76,8 @@ __host__ __device__ inline int64_t pow2_at_least(int64_t x) {
     return p;
 }
 
-// A tensor in alloc-step order, and in priority order (with its offset).
+// A tensor in alloc-step order, and in priority order (CTA tier; pos = its
+// alloc-order position).
 template <typename I>
 struct ARec {
     int64_t s;
@@ -68,21 +86,26 @@ struct ARec {
 template <typename I>
 struct SRec {
     int64_t s, off;
-    I a, f, id, pad;
+    I a, f, id, pos;
 };
 
+// Per-trace working set.  The records and the offsets (by alloc-order
+// position) share their bytes with the profile's difference array, which is
+// dead before the records are written.
 template <typename I>
 struct PlanLayout {
-    size_t arec, offid, bend, cst, lst, xl, dprof, total;
+    size_t arec, offp, dprof, bend, sb, lst, rp, total;
     __host__ __device__ PlanLayout(int64_t n, int64_t T, bool fused) {
         arec = 0;
-        offid = arec + align16((size_t)n * sizeof(ARec<I>));
-        bend = offid + align16((size_t)n * 8);
-        cst = bend + align16((size_t)T * 4);
-        lst = cst + align16((size_t)(n + 1) * 4);
-        xl = lst + align16((size_t)n * sizeof(I));
-        dprof = xl + align16((size_t)n * sizeof(I));
-        total = align_up(dprof + (fused ? align16(prof_padded((size_t)T) * 8) : 0));
+        offp = arec + align16((size_t)n * sizeof(ARec<I>));
+        const size_t main_end = offp + align16((size_t)n * 8);
+        dprof = 0;
+        const size_t dend = fused ? align16(prof_padded((size_t)T) * 8) : 0;
+        bend = main_end > dend ? main_end : dend;
+        sb = bend + align16((size_t)T * 4);
+        lst = sb + align16((size_t)((n + 31) / 32) * 4);
+        rp = lst + align16((size_t)n * 4);
+        total = align_up(rp + align16((size_t)n * 2));
     }
 };
 
@@ -153,55 +176,40 @@ __device__ __forceinline__ int64_t fit_best_scan(int64_t s, int64_t top, Each&& 
 
 // ------------------------------------------------------------- one thread
 
-// Places the component AR[p0, p0 + c), c <= kThreadComp, in registers; writes
-// offsets by id and returns the largest end.
+__device__ __forceinline__ int nib(uint32_t x, int k) { return (int)((x >> (4 * k)) & 15u); }
+
+// Places the component at alloc-order positions [p0, p0 + c), 2 <= c <=
+// kThreadComp, with one thread, from its members' precomputed ranks and
+// predecessor masks (RP[p] = rank | mask << 4); writes OFFP[p0 .. p0 + c) and
+// returns the largest end.
 template <typename I>
-__device__ int64_t place_thread(const ARec<I>* AR, int32_t p0, int32_t c, int32_t policy, int64_t* OFFID) {
-    int64_t s[kThreadComp], off[kThreadComp];
-    int32_t a[kThreadComp], f[kThreadComp], id[kThreadComp];
-#pragma unroll
-    for (int k = 0; k < kThreadComp; ++k) {
-        if (k < c) {
-            const ARec<I> r = AR[p0 + k];
-            s[k] = r.s;
-            a[k] = r.a;
-            f[k] = r.f;
-            id[k] = r.id;
-        } else {  // sentinel: after every real tensor
-            s[k] = -1;
-            a[k] = f[k] = 0;
-            id[k] = INT32_MAX;
-        }
-        off[k] = 0;
-    }
-    auto cx = [&](int x, int y) {  // order x before y by priority
-        const bool swap = s[y] != s[x] ? s[y] > s[x] : (a[y] != a[x] ? a[y] < a[x] : id[y] < id[x]);
-        if (swap) {
-            int64_t t64 = s[x]; s[x] = s[y]; s[y] = t64;
-            int32_t t = a[x]; a[x] = a[y]; a[y] = t;
-            t = f[x]; f[x] = f[y]; f[y] = t;
-            t = id[x]; id[x] = id[y]; id[y] = t;
-        }
-    };
-    cx(0, 1); cx(2, 3); cx(0, 2); cx(1, 3); cx(1, 2);  // sorting network for four
+__device__ int64_t place_thread(const ARec<I>* AR, const uint16_t* RP, int64_t* OFFP, int32_t p0, int32_t c,
+                                int32_t policy) {
+    static_assert(kThreadComp <= 8, "ranks are packed into 4-bit fields of 32 bits, masks into 12 bits");
+    uint32_t order = 0;  // field r = the member of rank r
+    for (int k = 0; k < c; ++k) order |= (uint32_t)k << (4 * (RP[p0 + k] & 15));
     int64_t mx = 0;
-#pragma unroll
-    for (int r = 0; r < kThreadComp; ++r) {
-        if (r >= c) break;
+    for (int r = 0; r < c; ++r) {
+        const int k = nib(order, r);
+        const uint32_t m = RP[p0 + k] >> 4;  // placed already: they precede it
+        const int64_t s = AR[p0 + k].s;
         auto each = [&](auto&& fn) {
-#pragma unroll
-            for (int q = 0; q < kThreadComp; ++q)
-                if (q < r && a[q] < f[r] && a[r] < f[q]) fn(off[q], off[q] + s[q]);
+            for (uint32_t t = m; t; t &= t - 1) {
+                const int q = __ffs(t) - 1;
+                const int64_t o = OFFP[p0 + q];
+                fn(o, o + AR[p0 + q].s);
+            }
         };
+        int64_t o;
         if (policy == MP_FIT_FIRST) {
-            off[r] = fit_first_scan(s[r], each);
+            o = fit_first_scan(s, each);
         } else {
             int64_t top = 0;
             each([&](int64_t, int64_t pe) { top = pe > top ? pe : top; });
-            off[r] = fit_best_scan(s[r], top, each);
+            o = fit_best_scan(s, top, each);
         }
-        OFFID[id[r]] = off[r];
-        mx = off[r] + s[r] > mx ? off[r] + s[r] : mx;
+        OFFP[p0 + k] = o;
+        mx = o + s > mx ? o + s : mx;
     }
     return mx;
 }
@@ -221,10 +229,11 @@ __device__ __forceinline__ int64_t warp_min_nonneg(int64_t v) {
     return (int64_t)(((uint64_t)hi << 32) | lo);
 }
 
-// Places the component AR[p0, p0 + c), c <= 32, with one warp (a tensor per
-// lane); every lane must call it.  Writes offsets by id; returns the largest end.
+// Places the component at positions [p0, p0 + c), c <= 32, with one warp (a
+// tensor per lane); every lane must call it.  Writes OFFP; returns the
+// largest end.
 template <typename I>
-__device__ int64_t place_warp(const ARec<I>* AR, int32_t p0, int32_t c, int32_t policy, int64_t* OFFID) {
+__device__ int64_t place_warp(const ARec<I>* AR, int64_t* OFFP, int32_t p0, int32_t c, int32_t policy) {
     const unsigned full = 0xffffffffu;
     const int lane = threadIdx.x & 31;
     const bool act = lane < c;
@@ -278,7 +287,7 @@ __device__ int64_t place_warp(const ARec<I>* AR, int32_t p0, int32_t c, int32_t 
             placed = true;
         }
     }
-    if (act) OFFID[id] = off;
+    if (act) OFFP[p0 + lane] = off;
     return warp_max_nonneg(act ? end : 0);
 }
 
@@ -447,15 +456,43 @@ __device__ void place_large(SRec<I>* R, int32_t c, int32_t policy, int64_t* bo, 
     }
 }
 
+// ------------------------------------------------------------- components
+
+// Size of the component starting at position p: distance to the next start
+// flag in SB (n positions, one bit each), or to n.
+__device__ __forceinline__ int32_t comp_size(const uint32_t* SB, int32_t p, int32_t n) {
+    int32_t w = p >> 5;
+    const int32_t nwords = (n + 31) >> 5;
+    uint32_t m = SB[w] & ~((2u << (p & 31)) - 1u);  // start flags after p in its word
+    while (m == 0) {
+        if (++w >= nwords) return n - p;
+        m = SB[w];
+    }
+    return (w << 5) + __ffs(m) - 1 - p;
+}
+
+// Size class of a component of c >= 2 tensors.
+__device__ __forceinline__ int comp_bin(int32_t c) {
+    return c > kWarpComp ? kBinCta : c > kThreadComp ? kBinWarp : kThreadComp - c;
+}
+
+// Position of step t in the padded difference array, in 32-bit arithmetic.
+__device__ __forceinline__ int32_t prof_pos32(int32_t t) {
+    return t + kProfPad * (int32_t)((uint32_t)t / kProfRun);
+}
+
+// ------------------------------------------------------------- the kernel
+
 template <typename I, bool kSmem, bool kFused>
 __global__ void __launch_bounds__(kSmem ? kPlanThreadsSmem : kPlanThreadsGlobal)
 k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_stride, size_t buf_offset,
        size_t buf_stride) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     __shared__ int64_t red[72];
-    __shared__ int32_t s_cnt, s_nt, s_nw, s_nx, s_bad;
+    __shared__ int32_t s_cnt, s_bin[kBins], s_base[kBins + 1], s_bad;
     __shared__ unsigned long long s_top, s_hi, s_lo, s_max, s_key, s_lbmax;
     const int b = blockIdx.x;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
     const int32_t policy = out.policy;
     int32_t* __restrict__ status = out.status;
     const bool want_profile = kFused && out.profile != nullptr;
@@ -468,29 +505,42 @@ k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_str
     const PlanLayout<I> L(kSmem ? n : bt.max_tensors, kSmem ? T : bt.max_steps, kFused);
     unsigned char* base = kSmem ? smem_raw : ws + (size_t)b * data_stride;
     ARec<I>* AR = reinterpret_cast<ARec<I>*>(base + L.arec);
-    int64_t* OFFID = reinterpret_cast<int64_t*>(base + L.offid);
+    int64_t* OFFP = reinterpret_cast<int64_t*>(base + L.offp);
+    int64_t* D = reinterpret_cast<int64_t*>(base + L.dprof);  // fused: before the records exist
     int32_t* BEND = reinterpret_cast<int32_t*>(base + L.bend);
-    int32_t* CST = reinterpret_cast<int32_t*>(base + L.cst);
-    I* LST = reinterpret_cast<I*>(base + L.lst);  // thread-tier components from the front, warp-tier from the back
-    I* XL = reinterpret_cast<I*>(base + L.xl);    // CTA-tier components
+    uint32_t* SB = reinterpret_cast<uint32_t*>(base + L.sb);
+    int32_t* LST = reinterpret_cast<int32_t*>(base + L.lst);
+    uint16_t* RP = reinterpret_cast<uint16_t*>(base + L.rp);
     // CTA tier workspace: predecessor offsets / ends, then the priority-ordered records
     const size_t cap2 = (size_t)pow2_at_least(bt.max_tensors > 0 ? bt.max_tensors : 1);
     int64_t* bo = reinterpret_cast<int64_t*>(ws + buf_offset + (size_t)b * buf_stride);
     int64_t* be = bo + cap2;
     SRec<I>* SR = reinterpret_cast<SRec<I>*>(be + cap2);
 
-    // ---- load, check, alloc-step histogram
+    // ---- clear the histogram (and the difference array)
     for (int t = threadIdx.x; t < T; t += blockDim.x) BEND[t] = 0;
+    const int32_t dlen = want_profile ? (int32_t)prof_padded((size_t)T) : 0;
+    for (int32_t t = threadIdx.x; t < dlen; t += blockDim.x) D[t] = 0;
+    if (threadIdx.x < kBins) s_bin[threadIdx.x] = 0;
     if (threadIdx.x == 0) {
-        s_nt = s_nw = s_nx = 0;
         s_bad = 0;
         s_hi = s_lo = s_max = s_lbmax = 0;
         s_key = ~0ull;
     }
     __syncthreads();
+
+    // ---- load, check, alloc-step histogram, profile differences.  The first
+    // kCached * blockDim tensors stay in registers for the scatter below.
     const int32_t* __restrict__ Ag = bt.alloc_step + tv.lo;
     const int32_t* __restrict__ Fg = bt.free_step + tv.lo;
     const int64_t* __restrict__ Sg = bt.size_bytes + tv.lo;
+    const bool vec = ((reinterpret_cast<uintptr_t>(Ag) | reinterpret_cast<uintptr_t>(Fg) |
+                       reinterpret_cast<uintptr_t>(Sg)) & 15) == 0;
+    auto cached_index = [&](int j) -> int32_t {
+        return vec ? 4 * (int32_t)threadIdx.x + j : (int32_t)threadIdx.x + j * (int32_t)blockDim.x;
+    };
+    int32_t ca[kCached], cf[kCached];
+    int64_t cs[kCached];
     bool ok = true;
     uint64_t sum = 0;
     auto take = [&](int32_t a, int32_t f, int64_t s) {
@@ -500,24 +550,35 @@ k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_str
         }
         sum = sat_add(sum, (uint64_t)s);
         atomicAdd(BEND + a, 1);
-    };
-    int k0 = 0;
-    if (((reinterpret_cast<uintptr_t>(Ag) | reinterpret_cast<uintptr_t>(Fg) | reinterpret_cast<uintptr_t>(Sg)) &
-         15) == 0) {
-        const int n4 = n >> 2;
-        for (int q = threadIdx.x; q < n4; q += blockDim.x) {
-            const int4 a = __ldg(reinterpret_cast<const int4*>(Ag) + q);
-            const int4 f = __ldg(reinterpret_cast<const int4*>(Fg) + q);
-            const longlong2 s01 = __ldg(reinterpret_cast<const longlong2*>(Sg) + 2 * q);
-            const longlong2 s23 = __ldg(reinterpret_cast<const longlong2*>(Sg) + 2 * q + 1);
-            take(a.x, f.x, s01.x);
-            take(a.y, f.y, s01.y);
-            take(a.z, f.z, s23.x);
-            take(a.w, f.w, s23.y);
+        if (want_profile) {
+            atomic_add_u64_split(D + prof_pos32(a), (uint64_t)s);
+            if (f < T) atomic_add_u64_split(D + prof_pos32(f), (uint64_t)(-s));
         }
-        k0 = n4 << 2;
+    };
+    if (vec && 4 * (int32_t)threadIdx.x + 3 < n) {
+        const int4 a = __ldg(reinterpret_cast<const int4*>(Ag) + threadIdx.x);
+        const int4 f = __ldg(reinterpret_cast<const int4*>(Fg) + threadIdx.x);
+        const longlong2 s01 = __ldg(reinterpret_cast<const longlong2*>(Sg) + 2 * threadIdx.x);
+        const longlong2 s23 = __ldg(reinterpret_cast<const longlong2*>(Sg) + 2 * threadIdx.x + 1);
+        ca[0] = a.x, ca[1] = a.y, ca[2] = a.z, ca[3] = a.w;
+        cf[0] = f.x, cf[1] = f.y, cf[2] = f.z, cf[3] = f.w;
+        cs[0] = s01.x, cs[1] = s01.y, cs[2] = s23.x, cs[3] = s23.y;
+    } else {
+#pragma unroll
+        for (int j = 0; j < kCached; ++j) {
+            const int32_t k = cached_index(j);
+            if (k < n) {
+                ca[j] = __ldg(Ag + k);
+                cf[j] = __ldg(Fg + k);
+                cs[j] = __ldg(Sg + k);
+            }
+        }
     }
-    for (int k = k0 + threadIdx.x; k < n; k += blockDim.x) take(__ldg(Ag + k), __ldg(Fg + k), __ldg(Sg + k));
+#pragma unroll
+    for (int j = 0; j < kCached; ++j)
+        if (cached_index(j) < n) take(ca[j], cf[j], cs[j]);
+    const int32_t nc = min(n, kCached * (int32_t)blockDim.x);
+    for (int32_t k = nc + threadIdx.x; k < n; k += blockDim.x) take(__ldg(Ag + k), __ldg(Fg + k), __ldg(Sg + k));
     block_add_size_sum(sum, &s_hi, &s_lo);
     if (!ok) s_bad = 1;
     __syncthreads();
@@ -530,42 +591,24 @@ k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_str
         return;
     }
 
-    // ---- counting sort into alloc-step records (second read hits the cache)
+    // ---- scan the histogram into bucket starts
     block_excl_scan_array<int32_t, 8>(BEND, T, reinterpret_cast<int32_t*>(red));
-    for (int k = threadIdx.x; k < n; k += blockDim.x) {
-        const int32_t a = __ldg(Ag + k);
-        ARec<I> r;
-        r.s = __ldg(Sg + k);
-        r.a = (I)a;
-        r.f = (I)__ldg(Fg + k);
-        r.id = (I)k;
-        r.pad = 0;
-        AR[atomicAdd(BEND + a, 1)] = r;
-    }
-    __syncthreads();
 
-    // ---- live profile from the records (fused): difference array, scan, write
+    // ---- live profile (fused): scan the difference array, write it out
     if (want_profile) {
-        int64_t* D = reinterpret_cast<int64_t*>(base + L.dprof);
-        const int64_t dlen = (int64_t)prof_padded((size_t)T);
-        for (int64_t t = threadIdx.x; t < dlen; t += blockDim.x) D[t] = 0;
-        __syncthreads();
-        for (int p = threadIdx.x; p < n; p += blockDim.x) {
-            const ARec<I> r = AR[p];
-            atomic_add_u64_split(D + prof_pos(r.a), (uint64_t)r.s);
-            if (r.f < T) atomic_add_u64_split(D + prof_pos(r.f), (uint64_t)(-r.s));
-        }
-        __syncthreads();
         int64_t* pout = out.profile + tv.plo;
         const bool vec_out = (reinterpret_cast<uintptr_t>(pout) & 15) == 0;
+        // kRun = kProfRun / 2 steps per lane: pairs of lanes share one padded
+        // run, and the 16-byte reads of eight lanes still cover all 32 banks
+        constexpr int kRun = kProfRun / 2;
         int64_t carry = 0, lmax = 0;
-        for (int64_t base_t = 0; base_t < T; base_t += (int64_t)blockDim.x * kProfRun) {
-            const int64_t my = base_t + (int64_t)threadIdx.x * kProfRun;
+        for (int64_t base_t = 0; base_t < T; base_t += (int64_t)blockDim.x * kRun) {
+            const int64_t my = base_t + (int64_t)threadIdx.x * kRun;
             const int64_t* run = D + prof_pos(my);
-            int64_t v[kProfRun];
+            int64_t v[kRun];
 #pragma unroll
-            for (int k = 0; k < kProfRun; k += 2) {
-                if (my + kProfRun <= T) {
+            for (int k = 0; k < kRun; k += 2) {
+                if (my + kRun <= T) {
                     const longlong2 q = *reinterpret_cast<const longlong2*>(run + k);
                     v[k] = q.x;
                     v[k + 1] = q.y;
@@ -575,86 +618,168 @@ k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_str
                 }
             }
 #pragma unroll
-            for (int k = 1; k < kProfRun; ++k) v[k] += v[k - 1];
+            for (int k = 1; k < kRun; ++k) v[k] += v[k - 1];
             int64_t tot;
-            const int64_t pre = block_excl_scan<int64_t>(v[kProfRun - 1], red, &tot) + carry;
+            const int64_t pre = block_excl_scan<int64_t>(v[kRun - 1], red, &tot) + carry;
 #pragma unroll
-            for (int k = 0; k < kProfRun; ++k) {
+            for (int k = 0; k < kRun; ++k) {
                 v[k] += pre;
                 lmax = v[k] > lmax ? v[k] : lmax;
             }
-            if (vec_out && my + kProfRun <= T) {
+            if (vec_out && my + kRun <= T) {
 #pragma unroll
-                for (int k = 0; k < kProfRun; k += 2)
+                for (int k = 0; k < kRun; k += 2)
                     *reinterpret_cast<longlong2*>(pout + my + k) = make_longlong2(v[k], v[k + 1]);
             } else {
 #pragma unroll
-                for (int k = 0; k < kProfRun; ++k)
+                for (int k = 0; k < kRun; ++k)
                     if (my + k < T) pout[my + k] = v[k];
             }
             carry += tot;
         }
         lmax = warp_max_i64(lmax);
-        if ((threadIdx.x & 31) == 0 && lmax > 0) atomicMax(&s_lbmax, (unsigned long long)lmax);
+        if (lane == 0 && lmax > 0) atomicMax(&s_lbmax, (unsigned long long)lmax);
+        __syncthreads();  // the difference array is dead from here on
     }
 
-    // ---- components: a run starts where no earlier tensor is live any more
-    const int32_t chunk = (n + blockDim.x - 1) / blockDim.x;
-    const int32_t q0 = min(n, (int32_t)threadIdx.x * chunk), q1 = min(n, q0 + chunk);
-    int64_t fmax = 0;
-    for (int32_t p = q0; p < q1; ++p) fmax = max(fmax, (int64_t)AR[p].f);
-    int64_t ftot;
-    const int64_t run0 = block_excl_max(fmax, red, &ftot);
-    int32_t starts = 0;
-    {
-        int64_t run = run0;
-        for (int32_t p = q0; p < q1; ++p) {
-            starts += (p == 0 || run <= AR[p].a) ? 1 : 0;
-            run = max(run, (int64_t)AR[p].f);
-        }
+    // ---- counting sort into alloc-step records; BEND[t] ends as the number
+    // of tensors with alloc step <= t
+    auto scatter = [&](int32_t k, int32_t a, int32_t f, int64_t s) {
+        ARec<I> r;
+        r.s = s;
+        r.a = (I)a;
+        r.f = (I)f;
+        r.id = (I)k;
+        r.pad = 0;
+        AR[atomicAdd(BEND + a, 1)] = r;
+    };
+#pragma unroll
+    for (int j = 0; j < kCached; ++j) {
+        const int32_t k = cached_index(j);
+        if (k < n) scatter(k, ca[j], cf[j], cs[j]);
     }
-    int32_t ncomp;
-    const int32_t first = block_excl_scan<int32_t>(starts, reinterpret_cast<int32_t*>(red), &ncomp);
-    {
-        int64_t run = run0;
-        int32_t idx = first;
-        for (int32_t p = q0; p < q1; ++p) {
-            if (p == 0 || run <= AR[p].a) CST[idx++] = p;
-            run = max(run, (int64_t)AR[p].f);
-        }
-    }
-    if (threadIdx.x == 0) CST[ncomp] = n;
+    for (int32_t k = nc + threadIdx.x; k < n; k += blockDim.x) scatter(k, __ldg(Ag + k), __ldg(Fg + k), __ldg(Sg + k));
     __syncthreads();
-    for (int32_t c = threadIdx.x; c < ncomp; c += blockDim.x) {
-        const int32_t sz = CST[c + 1] - CST[c];
-        if (sz <= kThreadComp) LST[atomicAdd(&s_nt, 1)] = (I)c;
-        else if (sz <= kWarpComp) LST[n - 1 - atomicAdd(&s_nw, 1)] = (I)c;
-        else XL[atomicAdd(&s_nx, 1)] = (I)c;
+
+    // ---- components: a run starts where no earlier tensor is live any more.
+    // Each warp scans a contiguous chunk of positions, 32 at a time.
+    const int32_t chunk = (((n + nwarps - 1) / nwarps) + 31) & ~31;
+    const int32_t w0 = min(n, warp * chunk), w1 = min(n, w0 + chunk);
+    {
+        unsigned fm = 0;
+        for (int32_t p = w0 + lane; p < w1; p += 32) fm = max(fm, (unsigned)AR[p].f);
+        fm = __reduce_max_sync(0xffffffffu, fm);
+        if (lane == 0) reinterpret_cast<int32_t*>(red)[warp] = (int32_t)fm;
+    }
+    __syncthreads();
+    {
+        int32_t carry = 0;
+        for (int k = 0; k < warp; ++k) carry = max(carry, reinterpret_cast<int32_t*>(red)[k]);
+        for (int32_t p0 = w0; p0 < w1; p0 += 32) {
+            const int32_t p = p0 + lane;
+            const bool valid = p < w1;
+            int32_t a = 0, f = 0;
+            if (valid) {
+                a = AR[p].a;
+                f = AR[p].f;
+            }
+            int32_t incl = f;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int32_t u = __shfl_up_sync(0xffffffffu, incl, o);
+                if (lane >= o) incl = max(incl, u);
+            }
+            int32_t excl = __shfl_up_sync(0xffffffffu, incl, 1);
+            excl = lane == 0 ? carry : max(carry, excl);
+            const unsigned starts = __ballot_sync(0xffffffffu, valid && (p == 0 || excl <= a));
+            if (lane == 0) SB[p0 >> 5] = starts;
+            carry = max(carry, __shfl_sync(0xffffffffu, incl, 31));
+        }
     }
     __syncthreads();
 
-    // ---- small and medium components: warps take the medium ones, then
-    // every thread the small ones
+    // ---- members, one thread per tensor: a single tensor is placed at 0; a
+    // member of a component of 2..kThreadComp tensors gets its rank and
+    // predecessor mask; component starts are counted by size class
     int64_t mx = 0;
-    {
-        const int32_t nw = s_nw, nt = s_nt, nwarps = blockDim.x >> 5;
-        for (int32_t k = threadIdx.x >> 5; k < nw; k += nwarps) {
-            const int32_t c = LST[n - 1 - k], p0 = CST[c];
-            const int64_t e = place_warp(AR, p0, CST[c + 1] - p0, policy, OFFID);
-            mx = e > mx ? e : mx;
+    const unsigned lt_mask = (1u << lane) - 1u;
+    for (int32_t q0 = 0; q0 < n; q0 += blockDim.x) {
+        const int32_t p = q0 + threadIdx.x;
+        int bin = -1;
+        if (p < n) {
+            int32_t w = p >> 5;
+            uint32_t m = SB[w] & (0xffffffffu >> (31 - (p & 31)));  // starts at or before p in its word
+            while (m == 0) m = SB[--w];                             // position 0 starts a component
+            const int32_t p0 = (w << 5) + 31 - __clz(m);
+            const int32_t c = comp_size(SB, p0, n);
+            if (c == 1) {
+                OFFP[p] = 0;
+                mx = max(mx, AR[p].s);
+            } else {
+                if (p == p0) bin = comp_bin(c);
+                if (c <= kThreadComp) {
+                    const ARec<I> me = AR[p];
+                    uint32_t rank = 0, pred = 0;
+                    for (int32_t j = 0; j < c; ++j) {
+                        const int32_t q = p0 + j;
+                        if (q == p) continue;
+                        const ARec<I> o = AR[q];
+                        const bool first = precedes(o, me);
+                        const bool ov = q < p ? (int32_t)o.f > (int32_t)me.a : (int32_t)o.a < (int32_t)me.f;
+                        rank += first ? 1u : 0u;
+                        pred |= (first && ov ? 1u : 0u) << j;
+                    }
+                    RP[p] = (uint16_t)(rank | (pred << 4));
+                }
+            }
         }
-        for (int32_t k = threadIdx.x; k < nt; k += blockDim.x) {
-            const int32_t c = LST[k], p0 = CST[c];
-            const int64_t e = place_thread(AR, p0, CST[c + 1] - p0, policy, OFFID);
-            mx = e > mx ? e : mx;
+        const unsigned grp = __match_any_sync(0xffffffffu, bin);
+        if (bin >= 0 && (grp & lt_mask) == 0) atomicAdd(&s_bin[bin], __popc(grp));
+    }
+    __syncthreads();
+    if (warp == 0) {  // class starts; s_bin becomes each class's cursor
+        const int32_t v = lane < kBins ? s_bin[lane] : 0;
+        const int32_t incl = warp_incl_scan(v);
+        if (lane < kBins) s_base[lane] = s_bin[lane] = incl - v;
+        if (lane == kBins - 1) s_base[kBins] = incl;
+    }
+    __syncthreads();
+    for (int32_t q0 = 0; q0 < n; q0 += blockDim.x) {
+        const int32_t p = q0 + threadIdx.x;
+        int bin = -1;
+        if (p < n && ((SB[p >> 5] >> (p & 31)) & 1u)) {
+            const int32_t c = comp_size(SB, p, n);
+            if (c > 1) bin = comp_bin(c);
+        }
+        const unsigned grp = __match_any_sync(0xffffffffu, bin);
+        const int leader = __ffs(grp) - 1;
+        int32_t at = 0;
+        if (bin >= 0 && lane == leader) at = atomicAdd(&s_bin[bin], __popc(grp));
+        at = __shfl_sync(0xffffffffu, at, leader);
+        if (bin >= 0) LST[at + __popc(grp & lt_mask)] = p;
+    }
+    __syncthreads();
+
+    // ---- warp tier, then the thread tier (largest first)
+    {
+        const int32_t wb = s_base[kBinWarp], nwc = s_base[kBinCta] - wb;
+        for (int32_t k = warp; k < nwc; k += nwarps) {
+            const int32_t p0 = LST[wb + k];
+            const int64_t e = place_warp(AR, OFFP, p0, comp_size(SB, p0, n), policy);
+            mx = max(mx, e);
+        }
+        for (int32_t g = threadIdx.x; g < wb; g += blockDim.x) {
+            const int32_t p0 = LST[g], c = comp_size(SB, p0, n);
+            const int64_t e = place_thread(AR, RP, OFFP, p0, c, policy);
+            mx = max(mx, e);
         }
     }
 
     // ---- large components, the whole CTA each
-    const int32_t nx = s_nx;
+    const int32_t xb = s_base[kBinCta], nx = s_base[kBins] - xb;
     const CtaScratch sc{red, &s_cnt, &s_top};
     for (int32_t q = 0; q < nx; ++q) {
-        const int32_t c = XL[q], p0 = CST[c], sz = CST[c + 1] - p0;
+        const int32_t p0 = LST[xb + q], sz = comp_size(SB, p0, n);
         const int32_t len = (int32_t)pow2_at_least(sz);
         int32_t* idx = reinterpret_cast<int32_t*>(bo);  // the index list lives in bo while sorting
         for (int32_t x = threadIdx.x; x < len; x += blockDim.x) idx[x] = x < sz ? p0 + x : -1;
@@ -663,44 +788,44 @@ k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_str
             return y < 0 ? x >= 0 : (x >= 0 && precedes(AR[x], AR[y]));
         });
         for (int32_t x = threadIdx.x; x < sz; x += blockDim.x) {
-            const ARec<I> me = AR[idx[x]];
-            SRec<I> out;
-            out.s = me.s;
-            out.off = 0;
-            out.a = me.a;
-            out.f = me.f;
-            out.id = me.id;
-            out.pad = 0;
-            SR[x] = out;
+            const int32_t p = idx[x];
+            const ARec<I> me = AR[p];
+            SRec<I> rec;
+            rec.s = me.s;
+            rec.off = 0;
+            rec.a = me.a;
+            rec.f = me.f;
+            rec.id = me.id;
+            rec.pos = (I)p;
+            SR[x] = rec;
         }
         __syncthreads();
         place_large(SR, sz, policy, bo, be, sc);
         for (int32_t x = threadIdx.x; x < sz; x += blockDim.x) {
             const int64_t o = SR[x].off;
-            OFFID[SR[x].id] = o;
-            mx = o + SR[x].s > mx ? o + SR[x].s : mx;
+            OFFP[SR[x].pos] = o;
+            mx = max(mx, o + SR[x].s);
         }
         __syncthreads();
     }
 
     mx = warp_max_i64(mx);
-    if ((threadIdx.x & 31) == 0 && mx > 0) atomicMax(&s_max, (unsigned long long)mx);
+    if (lane == 0 && mx > 0) atomicMax(&s_max, (unsigned long long)mx);
     __syncthreads();
 
     // ---- validation of the plan just made (fused): every lifetime-overlapping
     // pair once, from its earlier member in alloc order, is checked for address
     // overlap -- an independent pass over the alloc-ordered records
     if (kFused) {
-        for (int p = threadIdx.x; p < n; p += blockDim.x) {
+        for (int32_t p = threadIdx.x; p < n; p += blockDim.x) {
             const ARec<I> ri = AR[p];
             const int32_t stop = BEND[ri.f - 1];  // tensors with alloc < free_i
             if (stop <= p + 1) continue;
-            const int64_t oi = OFFID[ri.id], ei = oi + ri.s;
-            for (int q = p + 1; q < stop; ++q) {
-                const ARec<I> rj = AR[q];
-                const int64_t oj = OFFID[rj.id];
-                if (oi < oj + rj.s && oj < ei) {
-                    const uint32_t i = (uint32_t)ri.id, j = (uint32_t)rj.id;
+            const int64_t oi = OFFP[p], ei = oi + ri.s;
+            for (int32_t q = p + 1; q < stop; ++q) {
+                const int64_t oj = OFFP[q];
+                if (oi < oj + AR[q].s && oj < ei) {
+                    const uint32_t i = (uint32_t)ri.id, j = (uint32_t)AR[q].id;
                     atomicMin(&s_key, ((unsigned long long)(i < j ? i : j) << 32) | (i < j ? j : i));
                 }
             }
@@ -708,18 +833,19 @@ k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_str
         __syncthreads();
     }
 
-    // ---- outputs
-    for (int k = threadIdx.x; k < n; k += blockDim.x) out.offsets[tv.lo + k] = OFFID[k];
+    // ---- outputs (offsets by tensor id)
+    int64_t* __restrict__ offsets = out.offsets + tv.lo;
+    for (int32_t p = threadIdx.x; p < n; p += blockDim.x) offsets[(int32_t)AR[p].id] = OFFP[p];
     if (threadIdx.x == 0) {
         out.plan_peak[b] = (int64_t)s_max;
         if (kFused) {
             if (want_profile && out.peak_lb) out.peak_lb[b] = (int64_t)s_lbmax;
             const unsigned long long key = s_key;
-            const bool ok = key == ~0ull;
-            if (out.verdict) out.verdict[b] = ok ? 1 : 0;
+            const bool good = key == ~0ull;
+            if (out.verdict) out.verdict[b] = good ? 1 : 0;
             if (out.conflict) {
-                out.conflict[2 * b] = ok ? -1 : (int32_t)(key >> 32);
-                out.conflict[2 * b + 1] = ok ? -1 : (int32_t)(key & 0xffffffffu);
+                out.conflict[2 * b] = good ? -1 : (int32_t)(key >> 32);
+                out.conflict[2 * b + 1] = good ? -1 : (int32_t)(key & 0xffffffffu);
             }
         }
         status[b] = MP_OK;
