@@ -2,9 +2,12 @@
 //
 // Host-side argument checks, then one kernel launch per call on the caller's
 // stream.  No entry point allocates device memory or synchronises.
+#include <algorithm>
 #include <cstdint>
+#include <map>
 #include <mutex>
 #include <set>
+#include <tuple>
 #include <utility>
 
 #include "launch.h"
@@ -24,6 +27,27 @@ cudaError_t set_smem_limit(const void* func, size_t bytes) {
     e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemCeiling);
     if (e == cudaSuccess) done.insert({dev, func});
     return e;
+}
+
+cudaError_t max_resident_ctas(const void* func, int threads, size_t smem, int* ctas) {
+    static std::mutex mu;
+    static std::map<std::tuple<int, const void*, int, size_t>, int> cache;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    const auto key = std::make_tuple(dev, func, threads, smem);
+    std::lock_guard<std::mutex> lock(mu);
+    auto it = cache.find(key);
+    if (it == cache.end()) {
+        int sms = 0, per_sm = 0;
+        e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        if (e != cudaSuccess) return e;
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, func, threads, smem);
+        if (e != cudaSuccess) return e;
+        it = cache.emplace(key, std::max(1, sms * per_sm)).first;
+    }
+    *ctas = it->second;
+    return cudaSuccess;
 }
 
 }  // namespace mp

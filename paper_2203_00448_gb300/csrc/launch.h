@@ -26,6 +26,10 @@ constexpr size_t kPlanSmemLimit = kSmemCeiling;
 // Raises the kernel's dynamic shared memory ceiling once per device.
 cudaError_t set_smem_limit(const void* func, size_t bytes);
 
+// CTAs of `func` (threads, dynamic shared memory smem) the current device holds
+// at once: SM count x resident CTAs per SM (at least 1); cached per device.
+cudaError_t max_resident_ctas(const void* func, int threads, size_t smem, int* ctas);
+
 // Alignment of every workspace slice.
 constexpr size_t kAlign = 256;
 __host__ __device__ constexpr size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }

@@ -43,11 +43,20 @@
 // with block reductions; BEST by sorting the predecessors by offset and
 // scanning the running maximum end, which exposes every gap at once.
 //
+// Byte width.  Every offset the method produces is 0 or the end of another
+// tensor, so every offset, end and live-bytes value of a trace is at most the
+// sum of its sizes.  Each call therefore launches the kernel twice: first with
+// 32-bit byte arithmetic (W = uint32_t), which handles every trace whose sizes
+// sum below 2^32 and marks the others deferred; then with 64-bit arithmetic,
+// whose CTAs return at once unless their trace was deferred.
+//
 // Fused pass (mp_plan_and_validate): the difference array of the profile is
 // built while the inputs are first read, scanned and written out before the
 // records are scattered over the same shared memory; after placement every
 // lifetime-overlapping pair is checked once, from its earlier member in alloc
 // order, for address overlap.
+#include <algorithm>
+
 #include "common.cuh"
 #include "launch.h"
 
@@ -60,6 +69,7 @@ constexpr int32_t kWarpComp = 32;    // ... up to this size: one warp (a tensor 
 constexpr int32_t kCandMax = 64;     // CTA tier: up to this many predecessors, test all candidates
 constexpr int kCached = 4;           // tensors per thread kept in registers between the two input passes
 constexpr int64_t kNone = INT64_MAX;
+constexpr int32_t kDeferred = -1;    // trace status between the two launches: needs 64-bit bytes
 
 // Component size classes for the counting sort of the component list:
 // classes 0 .. kThreadComp - 2 hold sizes kThreadComp down to 2 (thread tier,
@@ -76,11 +86,39 @@ __host__ __device__ inline int64_t pow2_at_least(int64_t x) {
     return p;
 }
 
-// A tensor in alloc-step order, and in priority order (CTA tier; pos = its
-// alloc-order position).
-template <typename I>
+// Largest value of a byte word: "none" in minimum searches.
+template <typename W>
+__host__ __device__ constexpr W w_none() {
+    return sizeof(W) == 4 ? (W)UINT32_MAX : (W)INT64_MAX;
+}
+
+// Difference-array layout: runs of kRun entries, each followed by kPad
+// entries of padding, so that the 16-byte reads of eight lanes that scan
+// kLane consecutive steps each fall in distinct banks.
+template <typename W>
+struct ProfGeom;
+template <>
+struct ProfGeom<int64_t> {
+    static constexpr int kRun = 16, kPad = 2, kLane = 8;
+};
+template <>
+struct ProfGeom<uint32_t> {
+    static constexpr int kRun = 8, kPad = 4, kLane = 8;
+};
+template <typename W>
+__host__ __device__ constexpr int32_t dpos(int32_t t) {
+    return t + ProfGeom<W>::kPad * (int32_t)((uint32_t)t / ProfGeom<W>::kRun);
+}
+template <typename W>
+__host__ __device__ constexpr size_t dpadded(size_t T) {
+    return T + ProfGeom<W>::kPad * ((T + ProfGeom<W>::kRun - 1) / ProfGeom<W>::kRun);
+}
+
+// A tensor in alloc-step order; in priority order for the CTA tier (with its
+// alloc-order position), which always works in 64-bit bytes.
+template <typename I, typename W>
 struct ARec {
-    int64_t s;
+    W s;
     I a, f, id, pad;
 };
 template <typename I>
@@ -92,15 +130,15 @@ struct SRec {
 // Per-trace working set.  The records and the offsets (by alloc-order
 // position) share their bytes with the profile's difference array, which is
 // dead before the records are written.
-template <typename I>
+template <typename I, typename W>
 struct PlanLayout {
     size_t arec, offp, dprof, bend, sb, lst, rp, total;
     __host__ __device__ PlanLayout(int64_t n, int64_t T, bool fused) {
         arec = 0;
-        offp = arec + align16((size_t)n * sizeof(ARec<I>));
-        const size_t main_end = offp + align16((size_t)n * 8);
+        offp = arec + align16((size_t)n * sizeof(ARec<I, W>));
+        const size_t main_end = offp + align16((size_t)n * sizeof(W));
         dprof = 0;
-        const size_t dend = fused ? align16(prof_padded((size_t)T) * 8) : 0;
+        const size_t dend = fused ? align16(dpadded<W>((size_t)T) * sizeof(W)) : 0;
         bend = main_end > dend ? main_end : dend;
         sb = bend + align16((size_t)T * 4);
         lst = sb + align16((size_t)((n + 31) / 32) * 4);
@@ -133,12 +171,12 @@ __device__ __forceinline__ bool precedes(const R& x, const R& y) {
 // ------------------------------------------------------------- gap search
 
 // FIRST by jumping: `each(fn)` calls fn(off, end) for every predecessor.
-template <typename Each>
-__device__ __forceinline__ int64_t fit_first_scan(int64_t s, Each&& each) {
-    int64_t o = 0;
+template <typename W, typename Each>
+__device__ __forceinline__ W fit_first_scan(W s, Each&& each) {
+    W o = 0;
     for (;;) {
-        int64_t next = o;
-        each([&](int64_t po, int64_t pe) {
+        W next = o;
+        each([&](W po, W pe) {
             if (po < o + s && o < pe && pe > next) next = pe;
         });
         if (next == o) return o;
@@ -147,24 +185,24 @@ __device__ __forceinline__ int64_t fit_first_scan(int64_t s, Each&& each) {
 }
 
 // BEST by walking the free holes below the top in address order.
-template <typename Each>
-__device__ __forceinline__ int64_t fit_best_scan(int64_t s, int64_t top, Each&& each) {
-    int64_t c = 0, best_len = kNone, best = top;
+template <typename W, typename Each>
+__device__ __forceinline__ W fit_best_scan(W s, W top, Each&& each) {
+    W c = 0, best_len = w_none<W>(), best = top;
     while (c < top) {
         for (;;) {  // move c off any predecessor that covers it
-            int64_t next = c;
-            each([&](int64_t po, int64_t pe) {
+            W next = c;
+            each([&](W po, W pe) {
                 if (po <= c && c < pe && pe > next) next = pe;
             });
             if (next == c) break;
             c = next;
         }
         if (c >= top) break;
-        int64_t ns = kNone;  // c is uncovered and below the top: some start lies above it
-        each([&](int64_t po, int64_t) {
+        W ns = w_none<W>();  // c is uncovered and below the top: some start lies above it
+        each([&](W po, W) {
             if (po > c && po < ns) ns = po;
         });
-        const int64_t len = ns - c;
+        const W len = ns - c;
         if (len >= s && len < best_len) {
             best_len = len;
             best = c;
@@ -182,31 +220,31 @@ __device__ __forceinline__ int nib(uint32_t x, int k) { return (int)((x >> (4 * 
 // kThreadComp, with one thread, from its members' precomputed ranks and
 // predecessor masks (RP[p] = rank | mask << 4); writes OFFP[p0 .. p0 + c) and
 // returns the largest end.
-template <typename I>
-__device__ int64_t place_thread(const ARec<I>* AR, const uint16_t* RP, int64_t* OFFP, int32_t p0, int32_t c,
-                                int32_t policy) {
+template <typename I, typename W>
+__device__ W place_thread(const ARec<I, W>* AR, const uint16_t* RP, W* OFFP, int32_t p0, int32_t c,
+                          int32_t policy) {
     static_assert(kThreadComp <= 8, "ranks are packed into 4-bit fields of 32 bits, masks into 12 bits");
     uint32_t order = 0;  // field r = the member of rank r
     for (int k = 0; k < c; ++k) order |= (uint32_t)k << (4 * (RP[p0 + k] & 15));
-    int64_t mx = 0;
+    W mx = 0;
     for (int r = 0; r < c; ++r) {
         const int k = nib(order, r);
         const uint32_t m = RP[p0 + k] >> 4;  // placed already: they precede it
-        const int64_t s = AR[p0 + k].s;
+        const W s = AR[p0 + k].s;
         auto each = [&](auto&& fn) {
             for (uint32_t t = m; t; t &= t - 1) {
                 const int q = __ffs(t) - 1;
-                const int64_t o = OFFP[p0 + q];
+                const W o = OFFP[p0 + q];
                 fn(o, o + AR[p0 + q].s);
             }
         };
-        int64_t o;
+        W o;
         if (policy == MP_FIT_FIRST) {
-            o = fit_first_scan(s, each);
+            o = fit_first_scan<W>(s, each);
         } else {
-            int64_t top = 0;
-            each([&](int64_t, int64_t pe) { top = pe > top ? pe : top; });
-            o = fit_best_scan(s, top, each);
+            W top = 0;
+            each([&](W, W pe) { top = pe > top ? pe : top; });
+            o = fit_best_scan<W>(s, top, each);
         }
         OFFP[p0 + k] = o;
         mx = o + s > mx ? o + s : mx;
@@ -216,14 +254,17 @@ __device__ int64_t place_thread(const ARec<I>* AR, const uint16_t* RP, int64_t* 
 
 // ------------------------------------------------------------- one warp
 
-// Warp max / min of non-negative int64 values by two 32-bit reductions
-// (high words first, then the low words of the lanes holding the top high word).
-__device__ __forceinline__ int64_t warp_max_nonneg(int64_t v) {
+// Warp max / min of non-negative byte values: one 32-bit reduction, or two
+// for 64-bit values (high words first, then the low words of the lanes
+// holding the top high word).
+__device__ __forceinline__ uint32_t warp_max_w(uint32_t v) { return __reduce_max_sync(0xffffffffu, v); }
+__device__ __forceinline__ uint32_t warp_min_w(uint32_t v) { return __reduce_min_sync(0xffffffffu, v); }
+__device__ __forceinline__ int64_t warp_max_w(int64_t v) {
     const unsigned hi = __reduce_max_sync(0xffffffffu, (unsigned)((uint64_t)v >> 32));
     const unsigned lo = __reduce_max_sync(0xffffffffu, (unsigned)((uint64_t)v >> 32) == hi ? (unsigned)v : 0u);
     return (int64_t)(((uint64_t)hi << 32) | lo);
 }
-__device__ __forceinline__ int64_t warp_min_nonneg(int64_t v) {
+__device__ __forceinline__ int64_t warp_min_w(int64_t v) {
     const unsigned hi = __reduce_min_sync(0xffffffffu, (unsigned)((uint64_t)v >> 32));
     const unsigned lo = __reduce_min_sync(0xffffffffu, (unsigned)((uint64_t)v >> 32) == hi ? (unsigned)v : ~0u);
     return (int64_t)(((uint64_t)hi << 32) | lo);
@@ -232,48 +273,48 @@ __device__ __forceinline__ int64_t warp_min_nonneg(int64_t v) {
 // Places the component at positions [p0, p0 + c), c <= 32, with one warp (a
 // tensor per lane); every lane must call it.  Writes OFFP; returns the
 // largest end.
-template <typename I>
-__device__ int64_t place_warp(const ARec<I>* AR, int64_t* OFFP, int32_t p0, int32_t c, int32_t policy) {
+template <typename I, typename W>
+__device__ W place_warp(const ARec<I, W>* AR, W* OFFP, int32_t p0, int32_t c, int32_t policy) {
     const unsigned full = 0xffffffffu;
     const int lane = threadIdx.x & 31;
     const bool act = lane < c;
-    ARec<I> me;
+    ARec<I, W> me;
     if (act) me = AR[p0 + lane];
-    const int64_t s = act ? me.s : 0;
+    const W s = act ? me.s : 0;
     const int32_t a = act ? (int32_t)me.a : 0, f = act ? (int32_t)me.f : 0, id = act ? (int32_t)me.id : -1;
     int rank = 0;  // members that precede this one
     for (int l = 0; l < c; ++l) {
-        const int64_t sl = __shfl_sync(full, s, l);
+        const W sl = __shfl_sync(full, s, l);
         const int32_t al = __shfl_sync(full, a, l), il = __shfl_sync(full, id, l);
         if (act && l != lane) rank += (sl != s ? sl > s : (al != a ? al < a : il < id)) ? 1 : 0;
     }
-    int64_t off = 0, end = 0;
+    W off = 0, end = 0;
     bool placed = false;
     for (int r = 0; r < c; ++r) {
         const int src = __ffs(__ballot_sync(full, act && rank == r)) - 1;
         const int32_t ai = __shfl_sync(full, a, src), fi = __shfl_sync(full, f, src);
-        const int64_t si = __shfl_sync(full, s, src);
+        const W si = __shfl_sync(full, s, src);
         const bool pred = placed && a < fi && ai < f;  // placed: ranks below r
-        int64_t o = 0;
+        W o = 0;
         if (policy == MP_FIT_FIRST) {
             for (;;) {
-                const int64_t mx = warp_max_nonneg((pred && off < o + si && o < end) ? end : 0);
+                const W mx = warp_max_w((pred && off < o + si && o < end) ? end : (W)0);
                 if (mx <= o) break;
                 o = mx;
             }
         } else {
-            const int64_t top = warp_max_nonneg(pred ? end : 0);
-            int64_t cc = 0, best_len = kNone;
+            const W top = warp_max_w(pred ? end : (W)0);
+            W cc = 0, best_len = w_none<W>();
             o = top;
             while (cc < top) {
                 for (;;) {  // move cc off any predecessor that covers it
-                    const int64_t mx = warp_max_nonneg((pred && off <= cc && cc < end) ? end : 0);
+                    const W mx = warp_max_w((pred && off <= cc && cc < end) ? end : (W)0);
                     if (mx <= cc) break;
                     cc = mx;
                 }
                 if (cc >= top) break;
-                const int64_t ns = warp_min_nonneg((pred && off > cc) ? off : kNone);
-                const int64_t len = ns - cc;
+                const W ns = warp_min_w((pred && off > cc) ? off : w_none<W>());
+                const W len = ns - cc;
                 if (len >= si && len < best_len) {
                     best_len = len;
                     o = cc;
@@ -288,7 +329,7 @@ __device__ int64_t place_warp(const ARec<I>* AR, int64_t* OFFP, int32_t p0, int3
         }
     }
     if (act) OFFP[p0 + lane] = off;
-    return warp_max_nonneg(act ? end : 0);
+    return warp_max_w(act ? end : (W)0);
 }
 
 // ------------------------------------------------------------- whole CTA
@@ -476,22 +517,30 @@ __device__ __forceinline__ int comp_bin(int32_t c) {
     return c > kWarpComp ? kBinCta : c > kThreadComp ? kBinWarp : kThreadComp - c;
 }
 
-// Position of step t in the padded difference array, in 32-bit arithmetic.
-__device__ __forceinline__ int32_t prof_pos32(int32_t t) {
-    return t + kProfPad * (int32_t)((uint32_t)t / kProfRun);
+// Adds v into a difference-array entry: 64-bit as two 32-bit atomics, 32-bit
+// modulo 2^32 (exact once every add is in, since the true value fits).
+__device__ __forceinline__ void d_add(int64_t* d, int64_t v) { atomic_add_u64_split(d, (uint64_t)v); }
+__device__ __forceinline__ void d_add(uint32_t* d, int64_t v) { atomicAdd(d, (uint32_t)v); }
+
+// Block exclusive scan of one byte word per thread (uint32 words may not
+// wrap: every prefix of a trace's profile is below 2^32 on the 32-bit path).
+template <typename W>
+__device__ __forceinline__ W block_excl_scan_w(W v, int64_t* red, W* total) {
+    return block_excl_scan<W>(v, reinterpret_cast<W*>(red), total);
 }
 
 // ------------------------------------------------------------- the kernel
 
-template <typename I, bool kSmem, bool kFused>
-__global__ void __launch_bounds__(kSmem ? kPlanThreadsSmem : kPlanThreadsGlobal)
-k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_stride, size_t buf_offset,
-       size_t buf_stride) {
+// The whole path for trace b, by the whole CTA.
+template <typename I, typename W, bool kSmem, bool kFused>
+__device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, const PlanOut& out,
+                                           unsigned char* __restrict__ ws, size_t data_stride, size_t buf_offset,
+                                           size_t buf_stride) {
+    constexpr bool kWide = sizeof(W) == 8;
     extern __shared__ __align__(16) unsigned char smem_raw[];
     __shared__ int64_t red[72];
     __shared__ int32_t s_cnt, s_bin[kBins], s_base[kBins + 1], s_bad;
     __shared__ unsigned long long s_top, s_hi, s_lo, s_max, s_key, s_lbmax;
-    const int b = blockIdx.x;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
     const int32_t policy = out.policy;
     int32_t* __restrict__ status = out.status;
@@ -502,11 +551,11 @@ k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_str
         return;
     }
     const int32_t n = tv.n, T = tv.T;
-    const PlanLayout<I> L(kSmem ? n : bt.max_tensors, kSmem ? T : bt.max_steps, kFused);
+    const PlanLayout<I, W> L(kSmem ? n : bt.max_tensors, kSmem ? T : bt.max_steps, kFused);
     unsigned char* base = kSmem ? smem_raw : ws + (size_t)b * data_stride;
-    ARec<I>* AR = reinterpret_cast<ARec<I>*>(base + L.arec);
-    int64_t* OFFP = reinterpret_cast<int64_t*>(base + L.offp);
-    int64_t* D = reinterpret_cast<int64_t*>(base + L.dprof);  // fused: before the records exist
+    ARec<I, W>* AR = reinterpret_cast<ARec<I, W>*>(base + L.arec);
+    W* OFFP = reinterpret_cast<W*>(base + L.offp);
+    W* D = reinterpret_cast<W*>(base + L.dprof);  // fused: before the records exist
     int32_t* BEND = reinterpret_cast<int32_t*>(base + L.bend);
     uint32_t* SB = reinterpret_cast<uint32_t*>(base + L.sb);
     int32_t* LST = reinterpret_cast<int32_t*>(base + L.lst);
@@ -519,7 +568,7 @@ k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_str
 
     // ---- clear the histogram (and the difference array)
     for (int t = threadIdx.x; t < T; t += blockDim.x) BEND[t] = 0;
-    const int32_t dlen = want_profile ? (int32_t)prof_padded((size_t)T) : 0;
+    const int32_t dlen = want_profile ? (int32_t)dpadded<W>((size_t)T) : 0;
     for (int32_t t = threadIdx.x; t < dlen; t += blockDim.x) D[t] = 0;
     if (threadIdx.x < kBins) s_bin[threadIdx.x] = 0;
     if (threadIdx.x == 0) {
@@ -551,8 +600,8 @@ k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_str
         sum = sat_add(sum, (uint64_t)s);
         atomicAdd(BEND + a, 1);
         if (want_profile) {
-            atomic_add_u64_split(D + prof_pos32(a), (uint64_t)s);
-            if (f < T) atomic_add_u64_split(D + prof_pos32(f), (uint64_t)(-s));
+            d_add(D + dpos<W>(a), s);
+            if (f < T) d_add(D + dpos<W>(f), -s);
         }
     };
     if (vec && 4 * (int32_t)threadIdx.x + 3 < n) {
@@ -582,6 +631,10 @@ k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_str
     block_add_size_sum(sum, &s_hi, &s_lo);
     if (!ok) s_bad = 1;
     __syncthreads();
+    if (!kWide && !s_bad && (s_hi != 0 || s_lo > 0xffffffffull)) {  // sizes sum to 2^32 or more
+        if (threadIdx.x == 0) status[b] = kDeferred;
+        return;
+    }
     if (s_bad || size_sum_overflows(s_hi, s_lo)) {
         if (threadIdx.x == 0) {
             status[b] = s_bad ? MP_EINVAL : MP_EOVERFLOW;
@@ -598,29 +651,36 @@ k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_str
     if (want_profile) {
         int64_t* pout = out.profile + tv.plo;
         const bool vec_out = (reinterpret_cast<uintptr_t>(pout) & 15) == 0;
-        // kRun = kProfRun / 2 steps per lane: pairs of lanes share one padded
-        // run, and the 16-byte reads of eight lanes still cover all 32 banks
-        constexpr int kRun = kProfRun / 2;
-        int64_t carry = 0, lmax = 0;
-        for (int64_t base_t = 0; base_t < T; base_t += (int64_t)blockDim.x * kRun) {
-            const int64_t my = base_t + (int64_t)threadIdx.x * kRun;
-            const int64_t* run = D + prof_pos(my);
-            int64_t v[kRun];
+        constexpr int kRun = ProfGeom<W>::kLane;  // steps per lane and tile
+        constexpr int kVec = 16 / sizeof(W);      // words per 16-byte read
+        W carry = 0, lmax = 0;
+        for (int32_t base_t = 0; base_t < T; base_t += (int32_t)blockDim.x * kRun) {
+            const int32_t my = base_t + (int32_t)threadIdx.x * kRun;
+            const W* run = D + dpos<W>(my);
+            W v[kRun];
+            if (my + kRun <= T) {
 #pragma unroll
-            for (int k = 0; k < kRun; k += 2) {
-                if (my + kRun <= T) {
-                    const longlong2 q = *reinterpret_cast<const longlong2*>(run + k);
-                    v[k] = q.x;
-                    v[k + 1] = q.y;
-                } else {
-                    v[k] = my + k < T ? run[k] : 0;
-                    v[k + 1] = my + k + 1 < T ? run[k + 1] : 0;
+                for (int k = 0; k < kRun; k += kVec) {
+                    if constexpr (kWide) {
+                        const longlong2 q = *reinterpret_cast<const longlong2*>(run + k);
+                        v[k] = (W)q.x;
+                        v[k + 1] = (W)q.y;
+                    } else {
+                        const uint4 q = *reinterpret_cast<const uint4*>(run + k);
+                        v[k] = (W)q.x;
+                        v[k + 1] = (W)q.y;
+                        v[k + 2] = (W)q.z;
+                        v[k + 3] = (W)q.w;
+                    }
                 }
+            } else {
+#pragma unroll
+                for (int k = 0; k < kRun; ++k) v[k] = my + k < T ? run[k] : (W)0;
             }
 #pragma unroll
             for (int k = 1; k < kRun; ++k) v[k] += v[k - 1];
-            int64_t tot;
-            const int64_t pre = block_excl_scan<int64_t>(v[kRun - 1], red, &tot) + carry;
+            W tot;
+            const W pre = block_excl_scan_w<W>(v[kRun - 1], red, &tot) + carry;
 #pragma unroll
             for (int k = 0; k < kRun; ++k) {
                 v[k] += pre;
@@ -629,24 +689,24 @@ k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_str
             if (vec_out && my + kRun <= T) {
 #pragma unroll
                 for (int k = 0; k < kRun; k += 2)
-                    *reinterpret_cast<longlong2*>(pout + my + k) = make_longlong2(v[k], v[k + 1]);
+                    *reinterpret_cast<longlong2*>(pout + my + k) = make_longlong2((int64_t)v[k], (int64_t)v[k + 1]);
             } else {
 #pragma unroll
                 for (int k = 0; k < kRun; ++k)
-                    if (my + k < T) pout[my + k] = v[k];
+                    if (my + k < T) pout[my + k] = (int64_t)v[k];
             }
             carry += tot;
         }
-        lmax = warp_max_i64(lmax);
-        if (lane == 0 && lmax > 0) atomicMax(&s_lbmax, (unsigned long long)lmax);
+        const unsigned long long lm = (unsigned long long)warp_max_w(lmax);
+        if (lane == 0 && lm > 0) atomicMax(&s_lbmax, lm);
         __syncthreads();  // the difference array is dead from here on
     }
 
     // ---- counting sort into alloc-step records; BEND[t] ends as the number
     // of tensors with alloc step <= t
     auto scatter = [&](int32_t k, int32_t a, int32_t f, int64_t s) {
-        ARec<I> r;
-        r.s = s;
+        ARec<I, W> r;
+        r.s = (W)s;
         r.a = (I)a;
         r.f = (I)f;
         r.id = (I)k;
@@ -701,7 +761,7 @@ k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_str
     // ---- members, one thread per tensor: a single tensor is placed at 0; a
     // member of a component of 2..kThreadComp tensors gets its rank and
     // predecessor mask; component starts are counted by size class
-    int64_t mx = 0;
+    W mx = 0;
     const unsigned lt_mask = (1u << lane) - 1u;
     for (int32_t q0 = 0; q0 < n; q0 += blockDim.x) {
         const int32_t p = q0 + threadIdx.x;
@@ -718,12 +778,12 @@ k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_str
             } else {
                 if (p == p0) bin = comp_bin(c);
                 if (c <= kThreadComp) {
-                    const ARec<I> me = AR[p];
+                    const ARec<I, W> me = AR[p];
                     uint32_t rank = 0, pred = 0;
                     for (int32_t j = 0; j < c; ++j) {
                         const int32_t q = p0 + j;
                         if (q == p) continue;
-                        const ARec<I> o = AR[q];
+                        const ARec<I, W> o = AR[q];
                         const bool first = precedes(o, me);
                         const bool ov = q < p ? (int32_t)o.f > (int32_t)me.a : (int32_t)o.a < (int32_t)me.f;
                         rank += first ? 1u : 0u;
@@ -765,17 +825,17 @@ k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_str
         const int32_t wb = s_base[kBinWarp], nwc = s_base[kBinCta] - wb;
         for (int32_t k = warp; k < nwc; k += nwarps) {
             const int32_t p0 = LST[wb + k];
-            const int64_t e = place_warp(AR, OFFP, p0, comp_size(SB, p0, n), policy);
+            const W e = place_warp(AR, OFFP, p0, comp_size(SB, p0, n), policy);
             mx = max(mx, e);
         }
         for (int32_t g = threadIdx.x; g < wb; g += blockDim.x) {
             const int32_t p0 = LST[g], c = comp_size(SB, p0, n);
-            const int64_t e = place_thread(AR, RP, OFFP, p0, c, policy);
+            const W e = place_thread(AR, RP, OFFP, p0, c, policy);
             mx = max(mx, e);
         }
     }
 
-    // ---- large components, the whole CTA each
+    // ---- large components, the whole CTA each (64-bit bytes)
     const int32_t xb = s_base[kBinCta], nx = s_base[kBins] - xb;
     const CtaScratch sc{red, &s_cnt, &s_top};
     for (int32_t q = 0; q < nx; ++q) {
@@ -789,9 +849,9 @@ k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_str
         });
         for (int32_t x = threadIdx.x; x < sz; x += blockDim.x) {
             const int32_t p = idx[x];
-            const ARec<I> me = AR[p];
+            const ARec<I, W> me = AR[p];
             SRec<I> rec;
-            rec.s = me.s;
+            rec.s = (int64_t)me.s;
             rec.off = 0;
             rec.a = me.a;
             rec.f = me.f;
@@ -802,15 +862,17 @@ k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_str
         __syncthreads();
         place_large(SR, sz, policy, bo, be, sc);
         for (int32_t x = threadIdx.x; x < sz; x += blockDim.x) {
-            const int64_t o = SR[x].off;
+            const W o = (W)SR[x].off;
             OFFP[SR[x].pos] = o;
-            mx = max(mx, o + SR[x].s);
+            mx = max(mx, (W)(o + (W)SR[x].s));
         }
         __syncthreads();
     }
 
-    mx = warp_max_i64(mx);
-    if (lane == 0 && mx > 0) atomicMax(&s_max, (unsigned long long)mx);
+    {
+        const unsigned long long m = (unsigned long long)warp_max_w(mx);
+        if (lane == 0 && m > 0) atomicMax(&s_max, m);
+    }
     __syncthreads();
 
     // ---- validation of the plan just made (fused): every lifetime-overlapping
@@ -818,12 +880,12 @@ k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_str
     // overlap -- an independent pass over the alloc-ordered records
     if (kFused) {
         for (int32_t p = threadIdx.x; p < n; p += blockDim.x) {
-            const ARec<I> ri = AR[p];
+            const ARec<I, W> ri = AR[p];
             const int32_t stop = BEND[ri.f - 1];  // tensors with alloc < free_i
             if (stop <= p + 1) continue;
-            const int64_t oi = OFFP[p], ei = oi + ri.s;
+            const W oi = OFFP[p], ei = oi + ri.s;
             for (int32_t q = p + 1; q < stop; ++q) {
-                const int64_t oj = OFFP[q];
+                const W oj = OFFP[q];
                 if (oi < oj + AR[q].s && oj < ei) {
                     const uint32_t i = (uint32_t)ri.id, j = (uint32_t)AR[q].id;
                     atomicMin(&s_key, ((unsigned long long)(i < j ? i : j) << 32) | (i < j ? j : i));
@@ -835,7 +897,7 @@ k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_str
 
     // ---- outputs (offsets by tensor id)
     int64_t* __restrict__ offsets = out.offsets + tv.lo;
-    for (int32_t p = threadIdx.x; p < n; p += blockDim.x) offsets[(int32_t)AR[p].id] = OFFP[p];
+    for (int32_t p = threadIdx.x; p < n; p += blockDim.x) offsets[(int32_t)AR[p].id] = (int64_t)OFFP[p];
     if (threadIdx.x == 0) {
         out.plan_peak[b] = (int64_t)s_max;
         if (kFused) {
@@ -852,63 +914,111 @@ k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_str
     }
 }
 
+// 32-bit launch: one CTA per trace.  64-bit launch: a grid no larger than
+// what the GPU holds at once walks every trace and takes the ones the 32-bit
+// launch deferred.
+template <typename I, typename W, bool kSmem, bool kFused>
+__global__ void __launch_bounds__(kSmem ? kPlanThreadsSmem : kPlanThreadsGlobal)
+k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_stride, size_t buf_offset,
+       size_t buf_stride) {
+    if constexpr (sizeof(W) == 4) {
+        plan_trace<I, W, kSmem, kFused>(blockIdx.x, bt, out, ws, data_stride, buf_offset, buf_stride);
+    } else {
+        for (int b = blockIdx.x; b < bt.n_traces; b += gridDim.x) {
+            if (out.status[b] != kDeferred) continue;
+            plan_trace<I, W, kSmem, kFused>(b, bt, out, ws, data_stride, buf_offset, buf_stride);
+            __syncthreads();
+        }
+    }
+}
+
 struct PlanGeometry {
     bool smem, narrow;
-    size_t data, data_stride, buf_offset, buf_stride, workspace;
+    size_t data, data_stride;
 };
 
 // 16-bit indices when every id and step fits; shared memory when the trace's
-// working set fits under the ceiling, else a workspace slice per trace.  The
-// workspace always holds the CTA tier's buffers (predecessor offsets / ends,
-// the index list of a large component, and its records in priority order),
-// sized for up to max_tensors.
+// working set fits under the ceiling, else a workspace slice per trace.
+template <typename W>
 PlanGeometry plan_geometry(const mp_batch& bt, bool fused) {
     PlanGeometry g;
     g.narrow = bt.max_tensors < 32767 && bt.max_steps <= 32767;
-    g.data = g.narrow ? PlanLayout<int16_t>(bt.max_tensors, bt.max_steps, fused).total
-                      : PlanLayout<int32_t>(bt.max_tensors, bt.max_steps, fused).total;
+    g.data = g.narrow ? PlanLayout<int16_t, W>(bt.max_tensors, bt.max_steps, fused).total
+                      : PlanLayout<int32_t, W>(bt.max_tensors, bt.max_steps, fused).total;
     g.smem = g.data <= kPlanSmemLimit;
     g.data_stride = g.smem ? 0 : g.data;
-    g.buf_offset = (size_t)bt.n_traces * g.data_stride;
-    const size_t cap2 = (size_t)pow2_at_least(bt.max_tensors > 0 ? bt.max_tensors : 1);
-    g.buf_stride = align_up(cap2 * 16 + (size_t)bt.max_tensors * (g.narrow ? sizeof(SRec<int16_t>) : sizeof(SRec<int32_t>)));
-    g.workspace = bt.n_traces == 0 ? 0 : g.buf_offset + (size_t)bt.n_traces * g.buf_stride;
     return g;
 }
 
-template <typename I, bool kSmem, bool kFused>
-cudaError_t launch_variant(const mp_batch& bt, const PlanGeometry& g, const PlanOut& out, unsigned char* ws,
-                           cudaStream_t stream) {
+// Workspace: the per-trace slices of the launches that keep their data there
+// (the two launches run one after the other and share it), then the CTA
+// tier's buffers per trace (predecessor offsets / ends, the index list of a
+// large component, and its records in priority order), sized for up to
+// max_tensors.
+struct PlanWorkspace {
+    size_t buf_offset, buf_stride, total;
+};
+PlanWorkspace plan_workspace(const mp_batch& bt) {
+    PlanWorkspace w;
+    size_t slices = 0;
+    for (bool fused : {false, true}) {
+        const PlanGeometry a = plan_geometry<uint32_t>(bt, fused), b = plan_geometry<int64_t>(bt, fused);
+        slices = std::max(slices, std::max(a.data_stride, b.data_stride));
+    }
+    const bool narrow = bt.max_tensors < 32767 && bt.max_steps <= 32767;
+    const size_t cap2 = (size_t)pow2_at_least(bt.max_tensors > 0 ? bt.max_tensors : 1);
+    w.buf_offset = (size_t)bt.n_traces * slices;
+    w.buf_stride = align_up(cap2 * 16 + (size_t)bt.max_tensors * (narrow ? sizeof(SRec<int16_t>) : sizeof(SRec<int32_t>)));
+    w.total = bt.n_traces == 0 ? 0 : w.buf_offset + (size_t)bt.n_traces * w.buf_stride;
+    return w;
+}
+
+template <typename I, typename W, bool kSmem, bool kFused>
+cudaError_t launch_variant(const mp_batch& bt, const PlanGeometry& g, const PlanWorkspace& pw, const PlanOut& out,
+                           unsigned char* ws, cudaStream_t stream) {
     const size_t smem = kSmem ? g.data : 0;
+    const void* fn = (const void*)k_plan<I, W, kSmem, kFused>;
+    const int threads = kSmem ? kPlanThreadsSmem : kPlanThreadsGlobal;
     if (kSmem) {
-        cudaError_t e = set_smem_limit((const void*)k_plan<I, kSmem, kFused>, smem);
+        cudaError_t e = set_smem_limit(fn, smem);
         if (e != cudaSuccess) return e;
     }
-    k_plan<I, kSmem, kFused>
-        <<<(unsigned)bt.n_traces, kSmem ? kPlanThreadsSmem : kPlanThreadsGlobal, smem, stream>>>(
-            bt, out, ws, g.data_stride, g.buf_offset, g.buf_stride);
+    int grid = bt.n_traces;
+    if (sizeof(W) == 8) {
+        int resident = 0;
+        cudaError_t e = max_resident_ctas(fn, threads, smem, &resident);
+        if (e != cudaSuccess) return e;
+        grid = std::max(1, std::min(grid, resident));
+    }
+    k_plan<I, W, kSmem, kFused><<<(unsigned)grid, threads, smem, stream>>>(bt, out, ws, g.data_stride, pw.buf_offset,
+                                                                           pw.buf_stride);
     return cudaGetLastError();
+}
+
+template <typename W, bool kFused>
+cudaError_t launch_width(const mp_batch& bt, const PlanOut& out, unsigned char* ws, cudaStream_t stream) {
+    const PlanGeometry g = plan_geometry<W>(bt, kFused);
+    const PlanWorkspace pw = plan_workspace(bt);
+    if (g.narrow)
+        return g.smem ? launch_variant<int16_t, W, true, kFused>(bt, g, pw, out, ws, stream)
+                      : launch_variant<int16_t, W, false, kFused>(bt, g, pw, out, ws, stream);
+    return g.smem ? launch_variant<int32_t, W, true, kFused>(bt, g, pw, out, ws, stream)
+                  : launch_variant<int32_t, W, false, kFused>(bt, g, pw, out, ws, stream);
 }
 
 template <bool kFused>
 cudaError_t launch_any(const mp_batch& bt, const PlanOut& out, void* workspace, cudaStream_t stream) {
     if (bt.n_traces == 0) return cudaSuccess;
-    const PlanGeometry g = plan_geometry(bt, kFused);
     unsigned char* ws = static_cast<unsigned char*>(workspace);
-    if (g.narrow)
-        return g.smem ? launch_variant<int16_t, true, kFused>(bt, g, out, ws, stream)
-                      : launch_variant<int16_t, false, kFused>(bt, g, out, ws, stream);
-    return g.smem ? launch_variant<int32_t, true, kFused>(bt, g, out, ws, stream)
-                  : launch_variant<int32_t, false, kFused>(bt, g, out, ws, stream);
+    cudaError_t e = launch_width<uint32_t, kFused>(bt, out, ws, stream);
+    if (e != cudaSuccess) return e;
+    return launch_width<int64_t, kFused>(bt, out, ws, stream);
 }
 
 }  // namespace
 
 // One workspace size serves both the planner and the fused entry point.
-size_t plan_workspace_bytes(const mp_batch& bt) {
-    const size_t a = plan_geometry(bt, false).workspace, b = plan_geometry(bt, true).workspace;
-    return a > b ? a : b;
-}
+size_t plan_workspace_bytes(const mp_batch& bt) { return plan_workspace(bt).total; }
 
 cudaError_t launch_plan(const mp_batch& bt, int32_t policy, int64_t* offsets, int64_t* plan_peak,
                         int32_t* status, void* workspace, cudaStream_t stream) {

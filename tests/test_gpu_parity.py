@@ -272,3 +272,21 @@ def test_fused_without_profile(cuda_lib):
     ts = tg.config(2).select(range(0, 4096, 16))
     o = oracle_run(ts, oracle.FIT_FIRST)
     assert_fused_parity(ts, fused_run(ts, "first", profile=False), o, profile=False)
+
+
+def test_byte_width_boundary_and_mixed_batches(cuda_lib):
+    """Traces whose sizes sum just below, at and above 2^32 (the kernel switches
+    from 32-bit to 64-bit byte arithmetic there), interleaved with small ones in
+    one call, through both entry points."""
+    T, a, f, s = tg.config(0).trace(0)
+    traces = []
+    for target in (2 ** 32 - 1, 2 ** 32, 2 ** 32 + 1, 2 ** 33 + 12345):
+        s2 = np.asarray(s, dtype=np.int64).copy()
+        s2[0] += target - int(s2.sum())
+        traces += [(T, a, f, s2), tg.config(0).trace(0)]
+    ts = tg.from_arrays(traces)
+    for name, pol in POLICIES:
+        o = oracle_run(ts, pol)
+        assert (o["st"] == 0).all()
+        assert_parity(ts, gpu_run(ts, name), o)
+        assert_fused_parity(ts, fused_run(ts, name), o)
