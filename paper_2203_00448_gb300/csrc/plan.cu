@@ -918,7 +918,7 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
 // what the GPU holds at once walks every trace and takes the ones the 32-bit
 // launch deferred.
 template <typename I, typename W, bool kSmem, bool kFused>
-__global__ void __launch_bounds__(kSmem ? kPlanThreadsSmem : kPlanThreadsGlobal)
+__global__ void __launch_bounds__(kSmem ? kPlanThreadsSmem : kPlanThreadsGlobal, kSmem ? 9 : 1)
 k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_stride, size_t buf_offset,
        size_t buf_stride) {
     if constexpr (sizeof(W) == 4) {
