@@ -430,7 +430,8 @@ def run_gpu(args):
         "metric": METRIC, "value": total_tensors / (step_ms_max * 1e-3), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms_max, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
-        "config": {"workload": WORKLOAD_NAME, "n_traces": ts.n_traces * world, "tensors_per_trace": w["n"],
+        "config": {"workload": ts.name if world == 1 else WORKLOAD_NAME, "n_traces": ts.n_traces * world,
+                   "tensors_per_trace": w["n"],
                    "steps_per_trace": w["T"], "policy": args.policy,
                    "l2": "flushed before every timed step (256 MiB device write outside the timed events)",
                    "parallelism": f"dp{world} (traces sharded by rank, no collective)"},
