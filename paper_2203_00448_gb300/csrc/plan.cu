@@ -168,6 +168,19 @@ __device__ __forceinline__ bool precedes(const R& x, const R& y) {
     return x.id < y.id;
 }
 
+// The same order for 16-bit ids and steps and 32-bit sizes as one unsigned
+// key, smallest first: the complemented size, then the alloc step, then the id.
+template <typename R>
+__device__ __forceinline__ uint64_t prio_key(const R& r) {
+    return ((uint64_t)(~(uint32_t)r.s) << 32) | ((uint32_t)(uint16_t)r.a << 16) | (uint32_t)(uint16_t)r.id;
+}
+template <typename R>
+__device__ __forceinline__ bool precedes_key(const R& x, uint64_t key_y) {
+    constexpr bool kPacked = sizeof(x.s) == 4 && sizeof(x.a) == 2;
+    if constexpr (kPacked) return prio_key(x) < key_y;
+    return false;  // unused
+}
+
 // ------------------------------------------------------------- gap search
 
 // FIRST by jumping: `each(fn)` calls fn(off, end) for every predecessor.
@@ -779,12 +792,14 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
                 if (p == p0) bin = comp_bin(c);
                 if (c <= kThreadComp) {
                     const ARec<I, W> me = AR[p];
+                    constexpr bool kPacked = sizeof(W) == 4 && sizeof(I) == 2;
+                    const uint64_t me_key = kPacked ? prio_key(me) : 0;
                     uint32_t rank = 0, pred = 0;
                     for (int32_t j = 0; j < c; ++j) {
                         const int32_t q = p0 + j;
                         if (q == p) continue;
                         const ARec<I, W> o = AR[q];
-                        const bool first = precedes(o, me);
+                        const bool first = kPacked ? precedes_key(o, me_key) : precedes(o, me);
                         const bool ov = q < p ? (int32_t)o.f > (int32_t)me.a : (int32_t)o.a < (int32_t)me.f;
                         rank += first ? 1u : 0u;
                         pred |= (first && ov ? 1u : 0u) << j;
@@ -828,7 +843,9 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
             const W e = place_warp(AR, OFFP, p0, comp_size(SB, p0, n), policy);
             mx = max(mx, e);
         }
-        for (int32_t g = threadIdx.x; g < wb; g += blockDim.x) {
+        // the largest thread-tier components go to the last warp, which has
+        // the fewest warp-tier components
+        for (int32_t g = ((nwarps - 1 - warp) << 5) + lane; g < wb; g += blockDim.x) {
             const int32_t p0 = LST[g], c = comp_size(SB, p0, n);
             const W e = place_thread(AR, RP, OFFP, p0, c, policy);
             mx = max(mx, e);
