@@ -47,6 +47,8 @@ L2_FLUSH_BYTES = 256 << 20
 # fused   : read 16 B per tensor and 20 B per trace; write the profile 8 B per step,
 #           offsets 8 B per tensor, and peak_lb, plan_peak, verdict, conflict and
 #           status (32 B) per trace.
+# bump    : read 16 B per tensor and 12 B per trace; write offsets 8 B per tensor,
+#           plan_peak 8 B and status 4 B per trace.
 KERNELS = ("live_profile", "plan_greedy_by_size", "validate_plan")
 FUSED = "plan_and_validate"
 # mp_plan_and_validate launches the planner kernel twice: once with 32-bit byte
@@ -64,6 +66,8 @@ def algorithmic_bytes(kernel: str, n_tensors: int, n_traces: int, n_steps: int) 
         return 24 * n_tensors + (12 + 16) * n_traces
     if kernel == FUSED:
         return 24 * n_tensors + 8 * n_steps + (20 + 32) * n_traces
+    if kernel == "plan_bump":
+        return 24 * n_tensors + (12 + 12) * n_traces
     raise KeyError(kernel)
 
 
@@ -379,6 +383,28 @@ def run_gpu(args):
         torch.cuda.synchronize()
         per_kernel = [sum(ev[j].elapsed_time(ev[j + 1]) for ev in sep_events) / len(sep_events) for j in range(3)]
 
+    # Rows beyond the hot path, timed the same way on the same batch:
+    # bump_allocation (the baseline strategy of Sec. 2.3).
+    next_rows = None
+    if not args.no_breakdown:
+        bump_off = torch.empty_like(buf.offsets)
+        bump_pk = torch.empty_like(buf.plan_peak)
+        bump_st = torch.empty_like(buf.status[0])
+        for _ in range(args.warmup):
+            mp.plan_bump(db, bump_off, bump_pk, bump_st, stream=stream)
+        bump_events = [mk(2) for _ in range(max(3, args.steps // 2))]
+        for ev in bump_events:
+            flush.zero_()
+            ev[0].record(stream)
+            mp.plan_bump(db, bump_off, bump_pk, bump_st, stream=stream)
+            ev[1].record(stream)
+        torch.cuda.synchronize()
+        if not bool((bump_st == 0).all()):
+            print(json.dumps({"error": "plan_bump reported a failed trace", "rank": rank}))
+            return 1
+        bump_ms = sum(ev[0].elapsed_time(ev[1]) for ev in bump_events) / len(bump_events)
+        next_rows = {"plan_bump": {"ms": bump_ms}}
+
     # End to end through the host-buffer API: pinned H2D of the inputs, the
     # path, and D2H of every result, each step.
     e2e = None
@@ -409,6 +435,11 @@ def run_gpu(args):
         nbytes = algorithmic_bytes(name, ts.n_tensors, ts.n_traces, n_steps)
         gbs = nbytes / (per_kernel[j] * 1e-3) / 1e9
         kern[name] = {"ms": per_kernel[j], "algorithmic_bytes": nbytes, "achieved_gbs": gbs, "frac": gbs / peak}
+    if next_rows is not None:
+        for name, row in next_rows.items():
+            nbytes = algorithmic_bytes(name, ts.n_tensors, ts.n_traces, n_steps)
+            gbs = nbytes / (row["ms"] * 1e-3) / 1e9
+            row.update({"algorithmic_bytes": nbytes, "achieved_gbs": gbs, "frac": gbs / peak})
     fused_bytes = algorithmic_bytes(FUSED, ts.n_tensors, ts.n_traces, n_steps)
     fused_gbs = fused_bytes / (step_ms * 1e-3) / 1e9
     traffic = ncu_traffic(FUSED, ts.n_tensors)
@@ -440,6 +471,7 @@ def run_gpu(args):
         "gpu_launches": args.steps * LAUNCHES_PER_FUSED_CALL,
         "separate_kernels_ms_per_step": None if args.no_breakdown else sum(per_kernel),
         "separate_kernels": kern,
+        "next_rows": next_rows,
         "roofline": roof,
         "cpu_baseline": cpu_baseline,
         "e2e": e2e,

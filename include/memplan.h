@@ -190,6 +190,23 @@ mp_status mp_validate_plan(const mp_batch *batch, const int64_t *offsets, int32_
 mp_status mp_peak(const mp_batch *batch, const int64_t *offsets, int64_t *plan_peak,
                   int32_t *trace_status, void *stream);
 
+/* Bytes of device workspace mp_plan_bump needs for this batch (depends on the
+ * host scalars only).  0 means none. */
+size_t mp_bump_workspace_bytes(const mp_batch *batch);
+
+/* bump_allocation, the baseline strategy of Sec. 2.3: in allocation order
+ * (alloc_step ascending, then id ascending) every tensor is given the running
+ * offset, the sum of the sizes of the tensors allocated before it, so no
+ * address range is reused whatever the lifetimes.
+ * offsets[trace_ptr[b] + i]                                   int64[n_tensors]
+ * plan_peak[b] = the sum of the trace's sizes (its total_mem)   int64[B]
+ * trace_status[b]: MP_EINVAL / MP_EOVERFLOW as for mp_plan_greedy_by_size;
+ *   a failed trace gets plan_peak 0 and unspecified offsets.     int32[B]
+ * workspace: at least mp_bump_workspace_bytes(batch) bytes, rules as for
+ * mp_plan_greedy_by_size. */
+mp_status mp_plan_bump(const mp_batch *batch, int64_t *offsets, int64_t *plan_peak, int32_t *trace_status,
+                       void *workspace, size_t workspace_bytes, void *stream);
+
 /* Static, NUL-terminated name of a status code. */
 const char *mp_status_string(mp_status status);
 

@@ -5,15 +5,18 @@ include/memplan.h):
 
 1. live-bytes profile per op step and its peak lower bound;
 2. greedy_by_size offset assignment (first- or best-fit gaps) and the plan peak;
-3. pairwise validation of a plan against Eq. 2.1's ordering constraints.
+3. pairwise validation of a plan against Eq. 2.1's ordering constraints;
+
+and bump_allocation, the baseline strategy of Sec. 2.3.
 """
 from ._lib import (EINTERNAL, EINVAL, ENOMEM, EOVERFLOW, FIT_BEST, FIT_FIRST, OK, MemplanError,
                    status_string)
-from .api import (DeviceBatch, HostPath, PathBuffers, PathResult, Workspace, live_profile, peak, plan_and_validate, plan_greedy_by_size,
-                  plan_workspace_bytes, run_path, validate_plan, validate_workspace_bytes)
+from .api import (DeviceBatch, HostPath, PathBuffers, PathResult, Workspace, bump_workspace_bytes, live_profile, peak,
+                  plan_and_validate, plan_bump, plan_greedy_by_size, plan_workspace_bytes, run_path, validate_plan,
+                  validate_workspace_bytes)
 
 __all__ = [
-    "DeviceBatch", "HostPath", "PathBuffers", "PathResult", "Workspace", "live_profile", "peak", "plan_and_validate", "plan_greedy_by_size",
-    "plan_workspace_bytes", "run_path", "validate_plan", "validate_workspace_bytes", "MemplanError",
+    "DeviceBatch", "HostPath", "PathBuffers", "PathResult", "Workspace", "bump_workspace_bytes", "live_profile", "peak",
+    "plan_and_validate", "plan_bump", "plan_greedy_by_size", "plan_workspace_bytes", "run_path", "validate_plan", "validate_workspace_bytes", "MemplanError",
     "status_string", "OK", "EINVAL", "EOVERFLOW", "ENOMEM", "EINTERNAL", "FIT_FIRST", "FIT_BEST",
 ]

@@ -23,6 +23,8 @@ EXPORTS = (
     "mp_validate_workspace_bytes",
     "mp_validate_plan",
     "mp_peak",
+    "mp_bump_workspace_bytes",
+    "mp_plan_bump",
     "mp_status_string",
     "mp_abi_version",
 )
@@ -83,6 +85,10 @@ def load(path: str = LIB_PATH):
     lib.mp_validate_plan.restype = i32
     lib.mp_peak.argtypes = [BP, P, P, P, P]
     lib.mp_peak.restype = i32
+    lib.mp_bump_workspace_bytes.argtypes = [BP]
+    lib.mp_bump_workspace_bytes.restype = sz
+    lib.mp_plan_bump.argtypes = [BP, P, P, P, P, sz, P]
+    lib.mp_plan_bump.restype = i32
     lib.mp_status_string.argtypes = [i32]
     lib.mp_status_string.restype = ctypes.c_char_p
     lib.mp_abi_version.argtypes = []

@@ -205,6 +205,26 @@ def plan_and_validate(batch: DeviceBatch, policy="first", buffers: "PathBuffers 
                       buf.conflict.view(-1, 2), buf.status[0])
 
 
+def bump_workspace_bytes(batch: DeviceBatch) -> int:
+    s = batch.struct()
+    return int(_lib.load().mp_bump_workspace_bytes(ctypes.byref(s)))
+
+
+def plan_bump(batch: DeviceBatch, offsets=None, plan_peak=None, status=None, workspace: "Workspace | None" = None,
+              stream=None):
+    """bump_allocation (the baseline strategy of Sec. 2.3): each tensor at the
+    running offset in allocation order.  Returns (offsets, plan_peak, status)."""
+    lib, dev = _lib.load(), batch.device
+    offsets = _empty(batch.n_tensors, torch.int64, dev) if offsets is None else offsets
+    plan_peak = _empty(batch.n_traces, torch.int64, dev) if plan_peak is None else plan_peak
+    status = _empty(batch.n_traces, torch.int32, dev) if status is None else status
+    s = batch.struct()
+    wptr, wbytes = _workspace(workspace, dev).get(int(lib.mp_bump_workspace_bytes(ctypes.byref(s))))
+    _check("mp_plan_bump", lib.mp_plan_bump(ctypes.byref(s), _ptr(offsets), _ptr(plan_peak), _ptr(status), wptr,
+                                            wbytes, _stream_ptr(stream)))
+    return offsets, plan_peak, status
+
+
 def peak(batch: DeviceBatch, offsets: torch.Tensor, plan_peak=None, status=None, stream=None):
     """total_mem of a given plan per trace: max(offset + size)."""
     lib, dev = _lib.load(), batch.device

@@ -184,6 +184,25 @@ __attribute__((visibility("default"))) mp_status mp_validate_plan(const mp_batch
                                          static_cast<cudaStream_t>(stream)));
 }
 
+__attribute__((visibility("default"))) size_t mp_bump_workspace_bytes(const mp_batch* batch) {
+    if (check_batch(batch, false) != MP_OK) return 0;
+    return mp::bump_workspace_bytes(*batch);
+}
+
+__attribute__((visibility("default"))) mp_status mp_plan_bump(const mp_batch* batch, int64_t* offsets,
+                                                              int64_t* plan_peak, int32_t* trace_status,
+                                                              void* workspace, size_t workspace_bytes, void* stream) {
+    mp_status st = check_batch(batch, false);
+    if (st != MP_OK) return st;
+    if (!array_ok(offsets, batch->n_tensors) || !array_ok(plan_peak, batch->n_traces) ||
+        !array_ok(trace_status, batch->n_traces))
+        return MP_EINVAL;
+    st = check_workspace(mp::bump_workspace_bytes(*batch), workspace, workspace_bytes);
+    if (st != MP_OK) return st;
+    return from_cuda(mp::launch_bump(*batch, offsets, plan_peak, trace_status, workspace,
+                                     static_cast<cudaStream_t>(stream)));
+}
+
 __attribute__((visibility("default"))) mp_status mp_peak(const mp_batch* batch, const int64_t* offsets,
                                                          int64_t* plan_peak, int32_t* trace_status,
                                                          void* stream) {

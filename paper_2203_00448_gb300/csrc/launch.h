@@ -13,6 +13,7 @@ namespace mp {
 constexpr int kProfileThreads = 128;  // four traces per CTA, one warp each
 constexpr int kValidateThreads = 128;
 constexpr int kPeakThreads = 256;
+constexpr int kBumpThreads = 128;
 constexpr int kPlanThreadsSmem = 128;    // one CTA per trace, data in shared memory
 constexpr int kPlanThreadsGlobal = 1024; // one CTA per trace, data in the workspace
 
@@ -40,6 +41,10 @@ cudaError_t launch_live_profile(const mp_batch& bt, int64_t* profile, int64_t* p
 size_t validate_workspace_bytes(const mp_batch& bt);
 cudaError_t launch_validate(const mp_batch& bt, const int64_t* offsets, int32_t* verdict, int32_t* conflict,
                             int32_t* status, void* workspace, cudaStream_t stream);
+
+size_t bump_workspace_bytes(const mp_batch& bt);
+cudaError_t launch_bump(const mp_batch& bt, int64_t* offsets, int64_t* plan_peak, int32_t* status, void* workspace,
+                        cudaStream_t stream);
 
 cudaError_t launch_peak(const mp_batch& bt, const int64_t* offsets, int64_t* plan_peak, int32_t* status,
                         cudaStream_t stream);

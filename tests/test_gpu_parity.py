@@ -290,3 +290,34 @@ def test_byte_width_boundary_and_mixed_batches(cuda_lib):
         assert (o["st"] == 0).all()
         assert_parity(ts, gpu_run(ts, name), o)
         assert_fused_parity(ts, fused_run(ts, name), o)
+
+
+# ------------------------------------------------------------- bump_allocation
+
+def assert_bump_parity(ts):
+    import paper_2203_00448_gb300 as mp
+
+    db = mp.DeviceBatch.from_host(ts, "cuda")
+    off, pk, st = mp.plan_bump(db)
+    torch.cuda.synchronize()
+    o_off, o_pk, o_st = oracle.plan_bump(ts)
+    st, pk, off = st.cpu().numpy(), pk.cpu().numpy(), off.cpu().numpy()
+    assert np.array_equal(st, o_st), "trace status differs"
+    assert np.array_equal(pk, o_pk), "plan_peak differs"
+    for b in np.nonzero(o_st == 0)[0]:
+        lo, hi = ts.trace_ptr[b], ts.trace_ptr[b + 1]
+        assert np.array_equal(off[lo:hi], o_off[lo:hi]), f"offsets of trace {b}"
+
+
+@pytest.mark.parametrize("k", range(5))
+def test_bump_workload_parity(cuda_lib, k):
+    assert_bump_parity(tg.config(k))  # the long-tail trace keeps its working set in the workspace
+
+
+def test_bump_buckets_errors_and_ragged(cuda_lib):
+    rng = np.random.default_rng(3)
+    same_step = (50, np.zeros(300, np.int64), rng.integers(1, 51, 300), rng.integers(1, 1 << 20, 300))
+    for ts in (tg.random_small(21, 300, 120, 200, 1 << 20), tg.from_arrays([same_step, same_step]),
+               tg.from_tuples([(4, [(-1, 2, 8)]), (4, [(0, 1, 2 ** 62), (0, 2, 2 ** 62)]), (0, []), (5, []),
+                               (6, [(0, 3, 64), (1, 4, 32), (3, 6, 8), (1, 2, 16)])])):
+        assert_bump_parity(ts)
