@@ -8,6 +8,7 @@ collective on the data path).
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--policy first|best]
     python bench.py --impl reference ...   # the CPU oracle as the reference arm
+    python bench.py --all-configs          # every workload, one line each (not the bench line)
 
 Timing: W untimed warm-up steps; then K steps, each preceded by an L2 flush
 (256 MiB device write, outside the timed events) and timed with CUDA events
@@ -483,6 +484,77 @@ def run_gpu(args):
     return 0
 
 
+def _oracle_path(ts):
+    """Profile + plan (first fit) + validate of a TraceSet with the oracle; returns the seconds taken."""
+    import oracle
+
+    t0 = time.perf_counter()
+    oracle.live_profile(ts)
+    off, _, _ = oracle.plan_greedy_by_size(ts, oracle.FIT_FIRST)
+    oracle.validate_plan(ts, off)
+    return time.perf_counter() - t0
+
+
+def run_all_configs(args):
+    """Every workload of tracegen.CONFIG_NAMES through one mp_plan_and_validate
+    call, timed like the bench step, next to the oracle on 1 host core and on
+    all host cores (traces split over processes).  One JSON line per workload;
+    these are parity workloads with their own shapes, not the bench line."""
+    import multiprocessing as mproc
+
+    import torch
+
+    import paper_2203_00448_gb300 as mp
+    import tracegen
+    from paper_2203_00448_gb300 import build
+
+    cores = os.cpu_count() or 1
+    pool = mproc.get_context("spawn").Pool(cores)  # before the first GPU call
+    pool.map(_oracle_path, [tracegen.random_small(1, 2, 4, 8)] * cores)  # workers up and the oracle loaded
+    build.build()
+    dev = torch.device("cuda", torch.cuda.current_device())
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    peak, peak_kind = measured_peaks()
+    stream = torch.cuda.current_stream()
+    for k in sorted(tracegen.CONFIG_NAMES):
+        ts = tracegen.config(k)
+        db = mp.DeviceBatch.from_host(ts, dev)
+        buf = mp.PathBuffers(db)
+        for _ in range(args.warmup):
+            mp.plan_and_validate(db, args.policy, buf, stream=stream)
+        times = []
+        for _ in range(args.steps):
+            flush.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            mp.plan_and_validate(db, args.policy, buf, stream=stream)
+            e1.record(stream)
+            e1.synchronize()
+            times.append(e0.elapsed_time(e1))
+        ok = bool((buf.status[0] == 0).all()) and bool((buf.verdict == 1).all())
+        ms = statistics.median(times)
+        nbytes = algorithmic_bytes(FUSED, ts.n_tensors, ts.n_traces, ts.n_steps)
+        one_core = _oracle_path(ts)
+        n_chunks = min(cores, ts.n_traces)
+        chunks = [ts.select(range(c, ts.n_traces, n_chunks)) for c in range(n_chunks)]
+        t0 = time.perf_counter()
+        pool.map(_oracle_path, chunks)
+        all_cores = time.perf_counter() - t0
+        gbs = nbytes / (ms * 1e-3) / 1e9
+        print(json.dumps({
+            "workload": tracegen.CONFIG_NAMES[k], "policy": args.policy, "ok": ok, "n_traces": ts.n_traces,
+            "n_tensors": ts.n_tensors, "ms_per_call": ms, "tensors_per_s": ts.n_tensors / (ms * 1e-3),
+            "validated_pairs_per_s": ts.pairs() / (ms * 1e-3),
+            "roofline": {"bound": "hbm", "achieved": gbs, "peak": peak, "unit": "GB/s", "frac": gbs / peak,
+                         "peak_source": peak_kind, "algorithmic_bytes": nbytes},
+            "oracle_1core_s": one_core, "oracle_all_cores_s": all_cores, "oracle_cores": n_chunks,
+            "timing": f"median of {args.steps} calls after {args.warmup} warm-up, L2 flushed before each"}),
+            flush=True)
+    pool.close()
+    pool.join()
+    return 0
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -497,7 +569,11 @@ def main(argv=None):
                     help="skip the three-kernel breakdown (profiling runs that should launch the fused kernel only)")
     ap.add_argument("--traces", type=int, default=WORKLOAD["n_traces"],
                     help="traces per rank (the reported workload is the default 4096; other values are for profiling)")
+    ap.add_argument("--all-configs", action="store_true",
+                    help="time every workload (one JSON line each) beside the oracle on 1 and on all host cores")
     args = ap.parse_args(argv)
+    if args.all_configs:
+        return run_all_configs(args)
     if args.impl == "reference":
         return run_reference(args)
     return run_gpu(args)
