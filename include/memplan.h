@@ -207,6 +207,30 @@ size_t mp_bump_workspace_bytes(const mp_batch *batch);
 mp_status mp_plan_bump(const mp_batch *batch, int64_t *offsets, int64_t *plan_peak, int32_t *trace_status,
                        void *workspace, size_t workspace_bytes, void *stream);
 
+/* Traces of at most this many tensors are searched exhaustively by
+ * mp_plan_optimal. */
+#define MP_OPTIMAL_MAX_TENSORS 10
+
+/* Bytes of device workspace mp_plan_optimal needs for this batch (depends on
+ * the host scalars only). */
+size_t mp_optimal_workspace_bytes(const mp_batch *batch);
+
+/* The exact optimum of Eq. 2.1 (the smallest total_mem of any valid plan) for
+ * traces of at most MP_OPTIMAL_MAX_TENSORS tensors, by exhaustive search over
+ * every order of the tensors, each placed at its lowest feasible offset among
+ * the lifetime-overlapping tensors placed before it (some order reproduces any
+ * optimal packing).  It measures how far greedy_by_size is from optimal.
+ * offsets[trace_ptr[b] + i]: the plan of the first optimal order in
+ *   lexicographic order of tensor ids                        int64[n_tensors]
+ * opt_peak[b] = the optimum (0 for an empty trace)                int64[B]
+ * trace_status[b]: as for mp_plan_greedy_by_size; a trace of more than
+ *   MP_OPTIMAL_MAX_TENSORS tensors gets MP_EINVAL.                 int32[B]
+ * The search costs n! placements per trace of n tensors.
+ * workspace: at least mp_optimal_workspace_bytes(batch) bytes, rules as for
+ * mp_plan_greedy_by_size.  Two kernels are enqueued. */
+mp_status mp_plan_optimal(const mp_batch *batch, int64_t *offsets, int64_t *opt_peak, int32_t *trace_status,
+                          void *workspace, size_t workspace_bytes, void *stream);
+
 /* Static, NUL-terminated name of a status code. */
 const char *mp_status_string(mp_status status);
 

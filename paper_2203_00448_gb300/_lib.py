@@ -25,6 +25,8 @@ EXPORTS = (
     "mp_peak",
     "mp_bump_workspace_bytes",
     "mp_plan_bump",
+    "mp_optimal_workspace_bytes",
+    "mp_plan_optimal",
     "mp_status_string",
     "mp_abi_version",
 )
@@ -89,6 +91,10 @@ def load(path: str = LIB_PATH):
     lib.mp_bump_workspace_bytes.restype = sz
     lib.mp_plan_bump.argtypes = [BP, P, P, P, P, sz, P]
     lib.mp_plan_bump.restype = i32
+    lib.mp_optimal_workspace_bytes.argtypes = [BP]
+    lib.mp_optimal_workspace_bytes.restype = sz
+    lib.mp_plan_optimal.argtypes = [BP, P, P, P, P, sz, P]
+    lib.mp_plan_optimal.restype = i32
     lib.mp_status_string.argtypes = [i32]
     lib.mp_status_string.restype = ctypes.c_char_p
     lib.mp_abi_version.argtypes = []

@@ -225,6 +225,21 @@ def plan_bump(batch: DeviceBatch, offsets=None, plan_peak=None, status=None, wor
     return offsets, plan_peak, status
 
 
+def plan_optimal(batch: DeviceBatch, offsets=None, opt_peak=None, status=None, workspace: "Workspace | None" = None,
+                 stream=None):
+    """The exact optimum of Eq. 2.1 for traces of at most 10 tensors (exhaustive
+    search over tensor orders).  Returns (offsets, opt_peak, status)."""
+    lib, dev = _lib.load(), batch.device
+    offsets = _empty(batch.n_tensors, torch.int64, dev) if offsets is None else offsets
+    opt_peak = _empty(batch.n_traces, torch.int64, dev) if opt_peak is None else opt_peak
+    status = _empty(batch.n_traces, torch.int32, dev) if status is None else status
+    s = batch.struct()
+    wptr, wbytes = _workspace(workspace, dev).get(int(lib.mp_optimal_workspace_bytes(ctypes.byref(s))))
+    _check("mp_plan_optimal", lib.mp_plan_optimal(ctypes.byref(s), _ptr(offsets), _ptr(opt_peak), _ptr(status),
+                                                  wptr, wbytes, _stream_ptr(stream)))
+    return offsets, opt_peak, status
+
+
 def peak(batch: DeviceBatch, offsets: torch.Tensor, plan_peak=None, status=None, stream=None):
     """total_mem of a given plan per trace: max(offset + size)."""
     lib, dev = _lib.load(), batch.device

@@ -203,6 +203,28 @@ __attribute__((visibility("default"))) mp_status mp_plan_bump(const mp_batch* ba
                                      static_cast<cudaStream_t>(stream)));
 }
 
+__attribute__((visibility("default"))) size_t mp_optimal_workspace_bytes(const mp_batch* batch) {
+    if (check_batch(batch, false) != MP_OK) return 0;
+    return mp::optimal_workspace_bytes(*batch);
+}
+
+__attribute__((visibility("default"))) mp_status mp_plan_optimal(const mp_batch* batch, int64_t* offsets,
+                                                                 int64_t* opt_peak, int32_t* trace_status,
+                                                                 void* workspace, size_t workspace_bytes,
+                                                                 void* stream) {
+    mp_status st = check_batch(batch, false);
+    if (st != MP_OK) return st;
+    if (!array_ok(offsets, batch->n_tensors) || !array_ok(opt_peak, batch->n_traces) ||
+        !array_ok(trace_status, batch->n_traces))
+        return MP_EINVAL;
+    const size_t need = mp::optimal_workspace_bytes(*batch);
+    if (need > 0 && (int64_t)need / (int64_t)sizeof(longlong2) > INT32_MAX) return MP_EINVAL;  // grid too large
+    st = check_workspace(need, workspace, workspace_bytes);
+    if (st != MP_OK) return st;
+    return from_cuda(mp::launch_optimal(*batch, offsets, opt_peak, trace_status, workspace,
+                                        static_cast<cudaStream_t>(stream)));
+}
+
 __attribute__((visibility("default"))) mp_status mp_peak(const mp_batch* batch, const int64_t* offsets,
                                                          int64_t* plan_peak, int32_t* trace_status,
                                                          void* stream) {

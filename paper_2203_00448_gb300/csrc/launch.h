@@ -14,6 +14,7 @@ constexpr int kProfileThreads = 128;  // four traces per CTA, one warp each
 constexpr int kValidateThreads = 128;
 constexpr int kPeakThreads = 256;
 constexpr int kBumpThreads = 128;
+constexpr int kOptThreads = 128;
 constexpr int kPlanThreadsSmem = 128;    // one CTA per trace, data in shared memory
 constexpr int kPlanThreadsGlobal = 1024; // one CTA per trace, data in the workspace
 
@@ -45,6 +46,10 @@ cudaError_t launch_validate(const mp_batch& bt, const int64_t* offsets, int32_t*
 size_t bump_workspace_bytes(const mp_batch& bt);
 cudaError_t launch_bump(const mp_batch& bt, int64_t* offsets, int64_t* plan_peak, int32_t* status, void* workspace,
                         cudaStream_t stream);
+
+size_t optimal_workspace_bytes(const mp_batch& bt);
+cudaError_t launch_optimal(const mp_batch& bt, int64_t* offsets, int64_t* opt_peak, int32_t* status, void* workspace,
+                           cudaStream_t stream);
 
 cudaError_t launch_peak(const mp_batch& bt, const int64_t* offsets, int64_t* plan_peak, int32_t* status,
                         cudaStream_t stream);

@@ -321,3 +321,42 @@ def test_bump_buckets_errors_and_ragged(cuda_lib):
                tg.from_tuples([(4, [(-1, 2, 8)]), (4, [(0, 1, 2 ** 62), (0, 2, 2 ** 62)]), (0, []), (5, []),
                                (6, [(0, 3, 64), (1, 4, 32), (3, 6, 8), (1, 2, 16)])])):
         assert_bump_parity(ts)
+
+
+# ------------------------------------------------------------- exact optimum (small traces)
+
+def test_optimal_matches_oracle_brute_force(cuda_lib):
+    """mp_plan_optimal against the oracle's exhaustive search: the optimum and
+    the offsets of the first optimal order, on traces of 0..10 tensors with
+    few distinct sizes (many ties); lb <= opt <= greedy; more than 10 tensors
+    and invalid traces get their status codes."""
+    import paper_2203_00448_gb300 as mp
+
+    rng = np.random.default_rng(5)
+    traces = []
+    for n in (0, 1, 2, 3, 4, 5, 6, 7, 8, 8, 9, 9, 10, 6, 7):
+        T = int(rng.integers(1, 10))
+        a = rng.integers(0, T, n)
+        f = np.minimum(a + rng.integers(1, 5, n), T)
+        s = rng.integers(1, 5, n) * 64
+        traces.append((T, a, f, s))
+    big = traces[12]
+    traces += [(5, np.zeros(11, np.int64), np.full(11, 5), np.full(11, 8)),  # 11 tensors: beyond the search
+               (4, np.array([0, 2]), np.array([3, 1]), np.array([8, 8]))]     # free <= alloc
+    ts = tg.from_arrays(traces)
+    db = mp.DeviceBatch.from_host(ts, "cuda")
+    off, pk, st = mp.plan_optimal(db)
+    g_off, g_pk, g_st = mp.plan_greedy_by_size(db, "first")
+    torch.cuda.synchronize()
+    off, pk, st, g_pk = off.cpu().numpy(), pk.cpu().numpy(), st.cpu().numpy(), g_pk.cpu().numpy()
+    _, lb, _ = oracle.live_profile(ts)
+    assert list(st[-2:]) == [oracle.EINVAL, oracle.EINVAL]
+    for b in range(ts.n_traces - 2):
+        T, a, f, s = ts.trace(b)
+        assert st[b] == 0
+        opt, o_off = oracle.bruteforce_opt(a, f, s)
+        lo, hi = ts.trace_ptr[b], ts.trace_ptr[b + 1]
+        assert pk[b] == opt, f"trace {b}"
+        assert np.array_equal(off[lo:hi], o_off), f"offsets of trace {b}"
+        assert lb[b] <= opt <= g_pk[b]
+    assert len(big[1]) == 10
