@@ -405,6 +405,30 @@ def run_gpu(args):
             return 1
         bump_ms = sum(ev[0].elapsed_time(ev[1]) for ev in bump_events) / len(bump_events)
         next_rows = {"plan_bump": {"ms": bump_ms}}
+        # The exact optimum on small traces (the generator of the bench
+        # workload, 9 tensors over 6 steps, so that lifetimes overlap) and the
+        # gap of the greedy plan to it.
+        small = tracegen.random_batch(1 << 20, 4096, 9, 6, name="random-4096x9x6")
+        sdb = mp.DeviceBatch.from_host(small, dev)
+        ows = mp.Workspace(dev)
+        o_off, o_pk, o_st = mp.plan_optimal(sdb, workspace=ows, stream=stream)
+        g_off, g_pk, g_st = mp.plan_greedy_by_size(sdb, args.policy, stream=stream)
+        torch.cuda.synchronize()
+        opt_events = [mk(2) for _ in range(3)]
+        for ev in opt_events:
+            ev[0].record(stream)
+            mp.plan_optimal(sdb, o_off, o_pk, o_st, workspace=ows, stream=stream)
+            ev[1].record(stream)
+        torch.cuda.synchronize()
+        if not (bool((o_st == 0).all()) and bool((g_st == 0).all())):
+            print(json.dumps({"error": "plan_optimal reported a failed trace", "rank": rank}))
+            return 1
+        ratio = g_pk.double() / o_pk.double()
+        next_rows["plan_optimal"] = {
+            "ms": sum(ev[0].elapsed_time(ev[1]) for ev in opt_events) / len(opt_events),
+            "workload": small.name, "orders_per_trace": 362880,
+            "greedy_over_optimum": {"policy": args.policy, "mean": float(ratio.mean()), "max": float(ratio.max()),
+                                    "share_optimal": float((ratio == 1).double().mean())}}
 
     # End to end through the host-buffer API: pinned H2D of the inputs, the
     # path, and D2H of every result, each step.
@@ -438,6 +462,8 @@ def run_gpu(args):
         kern[name] = {"ms": per_kernel[j], "algorithmic_bytes": nbytes, "achieved_gbs": gbs, "frac": gbs / peak}
     if next_rows is not None:
         for name, row in next_rows.items():
+            if name != "plan_bump":
+                continue  # the exhaustive search is bound by its n! placements, not by memory
             nbytes = algorithmic_bytes(name, ts.n_tensors, ts.n_traces, n_steps)
             gbs = nbytes / (row["ms"] * 1e-3) / 1e9
             row.update({"algorithmic_bytes": nbytes, "achieved_gbs": gbs, "frac": gbs / peak})
