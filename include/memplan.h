@@ -231,6 +231,37 @@ size_t mp_optimal_workspace_bytes(const mp_batch *batch);
 mp_status mp_plan_optimal(const mp_batch *batch, int64_t *offsets, int64_t *opt_peak, int32_t *trace_status,
                           void *workspace, size_t workspace_bytes, void *stream);
 
+/* Alignment of every trace's slab placed by mp_slab_layout. */
+#define MP_SLAB_ALIGN 256
+
+/* Places one slab per trace in a single device buffer (Sec. 3.3:
+ * prim::AllocateSlab[total_size] per graph, every tensor a view at its
+ * offset): slab_base[b] = sum over earlier traces of plan_peak rounded up to
+ * MP_SLAB_ALIGN; slab_base[n_traces] = the buffer's size in bytes.
+ * plan_peak: int64[n_traces] device (negative values count as 0; give failed
+ * traces 0).  slab_base: int64[n_traces + 1] device.  One kernel. */
+mp_status mp_slab_layout(int32_t n_traces, const int64_t *plan_peak, int64_t *slab_base, void *stream);
+
+/* Bytes of device workspace mp_replay_plan needs for this batch. */
+size_t mp_replay_workspace_bytes(const mp_batch *batch);
+
+/* Replays each trace's plan on its slab, the check on real memory of Eq. 2.1:
+ * steps in order, at step t every tensor allocated at t fills its byte range
+ * [slab_base[b] + offset, + size) with a pattern of its own, then every tensor
+ * whose last live step is t (free = t + 1) compares its range with its
+ * pattern.  Two tensors that overlap in lifetime and in address make one of
+ * them fail, so ok[b] = 1 iff the plan is valid; first_bad[b] = the smallest id
+ * whose range was overwritten while it was live, or -1.
+ * slab: device buffer of slab_bytes bytes (4-byte aligned), for example sized
+ * by mp_slab_layout; its contents are overwritten.  Every tensor must lie in
+ * its trace's slab [0, slab_base[b+1] - slab_base[b]) and every slab in the
+ * buffer, else the trace gets MP_EINVAL and nothing of it is written.
+ * trace_status: as for mp_validate_plan.  workspace: at least
+ * mp_replay_workspace_bytes(batch) bytes. */
+mp_status mp_replay_plan(const mp_batch *batch, const int64_t *offsets, const int64_t *slab_base, void *slab,
+                         int64_t slab_bytes, int32_t *ok, int32_t *first_bad, int32_t *trace_status,
+                         void *workspace, size_t workspace_bytes, void *stream);
+
 /* Static, NUL-terminated name of a status code. */
 const char *mp_status_string(mp_status status);
 

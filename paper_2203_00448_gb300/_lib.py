@@ -27,6 +27,9 @@ EXPORTS = (
     "mp_plan_bump",
     "mp_optimal_workspace_bytes",
     "mp_plan_optimal",
+    "mp_slab_layout",
+    "mp_replay_workspace_bytes",
+    "mp_replay_plan",
     "mp_status_string",
     "mp_abi_version",
 )
@@ -95,6 +98,12 @@ def load(path: str = LIB_PATH):
     lib.mp_optimal_workspace_bytes.restype = sz
     lib.mp_plan_optimal.argtypes = [BP, P, P, P, P, sz, P]
     lib.mp_plan_optimal.restype = i32
+    lib.mp_slab_layout.argtypes = [i32, P, P, P]
+    lib.mp_slab_layout.restype = i32
+    lib.mp_replay_workspace_bytes.argtypes = [BP]
+    lib.mp_replay_workspace_bytes.restype = sz
+    lib.mp_replay_plan.argtypes = [BP, P, P, P, ctypes.c_int64, P, P, P, P, sz, P]
+    lib.mp_replay_plan.restype = i32
     lib.mp_status_string.argtypes = [i32]
     lib.mp_status_string.restype = ctypes.c_char_p
     lib.mp_abi_version.argtypes = []

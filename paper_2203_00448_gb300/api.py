@@ -240,6 +240,49 @@ def plan_optimal(batch: DeviceBatch, offsets=None, opt_peak=None, status=None, w
     return offsets, opt_peak, status
 
 
+def slab_layout(plan_peak: torch.Tensor, plan_status: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """Byte offset of every trace's slab in one buffer (Sec. 3.3's
+    prim::AllocateSlab per trace): int64[B + 1], the last entry the total.
+    Traces whose plan_status is non-zero get an empty slab."""
+    lib = _lib.load()
+    peaks = plan_peak if plan_status is None else torch.where(plan_status == 0, plan_peak, 0)
+    n = peaks.numel()
+    base = torch.empty(n + 1, dtype=torch.int64, device=peaks.device)
+    _check("mp_slab_layout", lib.mp_slab_layout(n, _ptr(peaks), base.data_ptr(), _stream_ptr(stream)))
+    return base
+
+
+def materialize(batch: DeviceBatch, offsets: torch.Tensor, plan_peak: torch.Tensor,
+                plan_status: torch.Tensor | None = None, stream=None):
+    """One device buffer holding every trace's slab, and every tensor's byte
+    address in it (Sec. 3.3's prim::AllocateTensor views): returns
+    (slab uint8 tensor, slab_base int64[B + 1], byte offset of each tensor in
+    the slab int64[n_tensors])."""
+    base = slab_layout(plan_peak, plan_status, stream)
+    total = int(base[-1].item())
+    slab = torch.empty(max(total, 1), dtype=torch.uint8, device=batch.device)
+    counts = batch.trace_ptr[1:] - batch.trace_ptr[:-1]
+    where = torch.repeat_interleave(base[:-1], counts) + offsets
+    return slab, base, where
+
+
+def replay_plan(batch: DeviceBatch, offsets: torch.Tensor, slab_base: torch.Tensor, slab: torch.Tensor,
+                workspace: "Workspace | None" = None, stream=None):
+    """Replays the plan on the slab (every tensor writes its pattern at its
+    alloc step and checks it at its last live step).  Returns (ok, first_bad,
+    status): ok[b] = 1 iff nothing was overwritten while live."""
+    lib, dev = _lib.load(), batch.device
+    ok = _empty(batch.n_traces, torch.int32, dev)
+    first_bad = _empty(batch.n_traces, torch.int32, dev)
+    status = _empty(batch.n_traces, torch.int32, dev)
+    s = batch.struct()
+    wptr, wbytes = _workspace(workspace, dev).get(int(lib.mp_replay_workspace_bytes(ctypes.byref(s))))
+    _check("mp_replay_plan", lib.mp_replay_plan(ctypes.byref(s), _ptr(offsets), _ptr(slab_base), slab.data_ptr(),
+                                                slab.numel(), _ptr(ok), _ptr(first_bad), _ptr(status), wptr, wbytes,
+                                                _stream_ptr(stream)))
+    return ok, first_bad, status
+
+
 def peak(batch: DeviceBatch, offsets: torch.Tensor, plan_peak=None, status=None, stream=None):
     """total_mem of a given plan per trace: max(offset + size)."""
     lib, dev = _lib.load(), batch.device

@@ -225,6 +225,36 @@ __attribute__((visibility("default"))) mp_status mp_plan_optimal(const mp_batch*
                                         static_cast<cudaStream_t>(stream)));
 }
 
+__attribute__((visibility("default"))) mp_status mp_slab_layout(int32_t n_traces, const int64_t* plan_peak,
+                                                                int64_t* slab_base, void* stream) {
+    if (n_traces < 0 || !array_ok(plan_peak, n_traces) || !array_ok(slab_base, (int64_t)n_traces + 1))
+        return MP_EINVAL;
+    return from_cuda(mp::launch_slab_layout(n_traces, plan_peak, slab_base, static_cast<cudaStream_t>(stream)));
+}
+
+__attribute__((visibility("default"))) size_t mp_replay_workspace_bytes(const mp_batch* batch) {
+    if (check_batch(batch, false) != MP_OK) return 0;
+    return mp::replay_workspace_bytes(*batch);
+}
+
+__attribute__((visibility("default"))) mp_status mp_replay_plan(const mp_batch* batch, const int64_t* offsets,
+                                                                const int64_t* slab_base, void* slab,
+                                                                int64_t slab_bytes, int32_t* ok, int32_t* first_bad,
+                                                                int32_t* trace_status, void* workspace,
+                                                                size_t workspace_bytes, void* stream) {
+    mp_status st = check_batch(batch, false);
+    if (st != MP_OK) return st;
+    if (!array_ok(offsets, batch->n_tensors) || !array_ok(slab_base, batch->n_traces ? batch->n_traces + 1 : 0) ||
+        !array_ok(ok, batch->n_traces) || !array_ok(first_bad, batch->n_traces) ||
+        !array_ok(trace_status, batch->n_traces) || slab_bytes < 0 ||
+        !array_ok(static_cast<const int32_t*>(slab), slab_bytes > 0 ? 1 : 0))
+        return MP_EINVAL;
+    st = check_workspace(mp::replay_workspace_bytes(*batch), workspace, workspace_bytes);
+    if (st != MP_OK) return st;
+    return from_cuda(mp::launch_replay(*batch, offsets, slab_base, static_cast<unsigned char*>(slab), slab_bytes, ok,
+                                       first_bad, trace_status, workspace, static_cast<cudaStream_t>(stream)));
+}
+
 __attribute__((visibility("default"))) mp_status mp_peak(const mp_batch* batch, const int64_t* offsets,
                                                          int64_t* plan_peak, int32_t* trace_status,
                                                          void* stream) {

@@ -360,3 +360,61 @@ def test_optimal_matches_oracle_brute_force(cuda_lib):
         assert np.array_equal(off[lo:hi], o_off), f"offsets of trace {b}"
         assert lb[b] <= opt <= g_pk[b]
     assert len(big[1]) == 10
+
+
+# ------------------------------------------------------------- plans replayed on device memory
+
+def test_replay_on_device_slabs(cuda_lib):
+    """Plans materialised on one device buffer (a slab per trace) and replayed:
+    greedy and bump plans replay cleanly; plans with a planted address clash
+    between lifetime-overlapping tensors fail exactly where the validator says
+    so; a tensor outside its slab is rejected before anything is written."""
+    import paper_2203_00448_gb300 as mp
+
+    ts = tg.from_arrays([tg.config(0).trace(0), tg.config(1).trace(0)] +
+                        [tg.config(2).trace(b) for b in range(0, 4096, 128)] +
+                        [tg.random_small(31, 1, 60, 40, 1 << 12).trace(0), (3, [], [], [])])
+    db = mp.DeviceBatch.from_host(ts, "cuda")
+    for plan in (lambda: mp.plan_greedy_by_size(db, "first"), lambda: mp.plan_greedy_by_size(db, "best"),
+                 lambda: mp.plan_bump(db)):
+        off, pk, st = plan()
+        slab, base, where = mp.materialize(db, off, pk, st)
+        ok, first_bad, rst = mp.replay_plan(db, off, base, slab)
+        torch.cuda.synchronize()
+        assert bool((rst == 0).all()) and bool((ok == 1).all()) and bool((first_bad == -1).all())
+        assert int(base[-1]) >= int(pk.sum())
+
+    # planted clashes: in every other trace, one tensor moved onto a lifetime-overlapping one
+    off, _, _ = mp.plan_greedy_by_size(db, "first")
+    h = off.cpu().numpy().copy()
+    rng = np.random.default_rng(9)
+    for b in range(0, ts.n_traces, 2):
+        T, a, f, s = ts.trace(b)
+        pairs = [(i, j) for i in range(len(a)) for j in range(len(a)) if i != j and a[i] < f[j] and a[j] < f[i]]
+        if pairs:
+            i, j = pairs[int(rng.integers(len(pairs)))]
+            h[ts.trace_ptr[b] + j] = h[ts.trace_ptr[b] + i]
+    bad_off = torch.from_numpy(h).cuda()
+    pk2, st2 = mp.peak(db, bad_off)
+    verdict, _, vst = mp.validate_plan(db, bad_off)
+    slab, base, _ = mp.materialize(db, bad_off, pk2, st2)
+    ok, first_bad, rst = mp.replay_plan(db, bad_off, base, slab)
+    torch.cuda.synchronize()
+    assert bool((rst == 0).all()) and bool((vst == 0).all())
+    assert torch.equal(ok, verdict)
+    assert int((verdict == 0).sum()) >= 10
+    fb = first_bad.cpu().numpy()
+    assert all((fb[b] >= 0) == (int(verdict[b]) == 0) for b in range(ts.n_traces))
+
+    # a tensor past its trace's slab, and a buffer too small for the last slabs
+    off, pk, st = mp.plan_greedy_by_size(db, "first")
+    slab, base, _ = mp.materialize(db, off, pk, st)
+    h = off.cpu().numpy().copy()
+    h[ts.trace_ptr[1]] = int(pk[1]) + 1
+    ok, _, rst = mp.replay_plan(db, torch.from_numpy(h).cuda(), base, slab)
+    short = slab[: int(base[3])]
+    ok2, _, rst2 = mp.replay_plan(db, off, base, short)
+    torch.cuda.synchronize()
+    assert int(rst[1]) == oracle.EINVAL and int(ok[1]) == 0 and bool((rst[2:] == 0).all())
+    r2 = rst2.cpu().numpy()
+    assert (r2[:3] == 0).all() and (r2[3:][np.diff(base.cpu().numpy())[3:] > 0] == oracle.EINVAL).all()
