@@ -86,6 +86,14 @@ class DeviceBatch:
     def device(self) -> torch.device:
         return self.alloc_step.device
 
+    def slice_traces(self, t0: int, t1: int) -> "DeviceBatch":
+        """The traces [t0, t1) as a batch of their own, sharing this batch's
+        device arrays (the CSR offsets stay global, so per-tensor and per-step
+        outputs keep their positions)."""
+        return DeviceBatch(self.trace_ptr[t0:t1 + 1], self.steps[t0:t1], self.profile_ptr[t0:t1 + 1],
+                           self.alloc_step, self.free_step, self.size_bytes, t1 - t0, self.max_tensors,
+                           self.max_steps, self.n_tensors, self.n_steps)
+
     def struct(self) -> MpBatch:
         return MpBatch(self.n_traces, self.max_tensors, self.max_steps, 0, self.n_tensors, self.n_steps,
                        _ptr(self.trace_ptr), _ptr(self.steps), _ptr(self.profile_ptr), _ptr(self.alloc_step),
@@ -323,6 +331,16 @@ class PathBuffers:
         self.plan_ws.get(plan_workspace_bytes(batch))
         self.validate_ws.get(validate_workspace_bytes(batch))
 
+    def slice_traces(self, t0: int, t1: int) -> "PathBuffers":
+        """Views of the outputs for traces [t0, t1) (profile and offsets whole,
+        as their positions are global), sharing the workspaces."""
+        v = object.__new__(PathBuffers)
+        v.profile, v.offsets = self.profile, self.offsets
+        v.peak_lb, v.plan_peak, v.verdict = self.peak_lb[t0:t1], self.plan_peak[t0:t1], self.verdict[t0:t1]
+        v.conflict, v.status = self.conflict[2 * t0:2 * t1], self.status[:, t0:t1]
+        v.plan_ws, v.validate_ws = self.plan_ws, self.validate_ws
+        return v
+
 
 def run_path(batch: DeviceBatch, policy="first", buffers: PathBuffers | None = None, stream=None) -> PathResult:
     """One pass of the whole path: profile, greedy_by_size plan (with its peak), validation."""
@@ -336,41 +354,78 @@ def run_path(batch: DeviceBatch, policy="first", buffers: PathBuffers | None = N
                       buf.conflict.view(-1, 2), buf.status)
 
 
+def _packed(specs, device=None, pin_memory=False):
+    """One byte buffer holding the named arrays (each start 16-byte aligned),
+    and a typed view of each: returns (buffer, {name: view})."""
+    starts, pos = [], 0
+    for _, shape, dt in specs:
+        pos = (pos + 15) & ~15
+        starts.append(pos)
+        pos += int(torch.Size(shape).numel()) * torch.empty((), dtype=dt).element_size()
+    buf = torch.empty(max(pos, 16), dtype=torch.uint8, device=device, pin_memory=pin_memory)
+    views = {}
+    for (name, shape, dt), o in zip(specs, starts):
+        nbytes = int(torch.Size(shape).numel()) * torch.empty((), dtype=dt).element_size()
+        views[name] = buf[o:o + nbytes].view(dt).view(shape)
+    return buf, views
+
+
 class HostPath:
-    """End-to-end use from host memory: copies a batch from pinned host buffers
+    """End-to-end use from host memory: copies a batch from pinned host memory
     to the device, runs the whole path (one plan_and_validate call), and copies
     every result back.
+
+    Inputs and outputs each live in one device buffer mirrored by one pinned
+    host buffer of the same layout, so a run is one copy in, the fused call
+    and one copy out.
 
     ``run(ts)`` takes a host batch (numpy arrays, e.g. tracegen.TraceSet) with
     the same shape as the one the object was built for and returns host
     numpy views of profile, peak_lb, offsets, plan_peak, verdict, conflict,
-    status.  All copies are stream-ordered on the given stream.
+    status.  All work is on the given (or current) stream; run() returns once
+    the results are on the host.
     """
 
     _IN = ("trace_ptr", "steps", "profile_ptr", "alloc_step", "free_step", "size_bytes")
+    _OUT = ("profile", "peak_lb", "offsets", "plan_peak", "verdict", "conflict", "status")
 
     def __init__(self, ts, device="cuda", policy="first", stream=None):
         self.policy = policy
         self.stream = stream
-        self.dev_batch = DeviceBatch.from_host(ts, device)
-        self.buffers = PathBuffers(self.dev_batch)
-        self.host_in = {k: torch.empty(tuple(getattr(self.dev_batch, k).shape), dtype=getattr(self.dev_batch, k).dtype,
-                                       pin_memory=True) for k in self._IN}
-        self._outs = ("profile", "peak_lb", "offsets", "plan_peak", "verdict", "conflict", "status")
-        shape = lambda k: tuple(getattr(self.buffers, k).shape[1:] if k == "status" else getattr(self.buffers, k).shape)
-        self.host_out = {k: torch.empty(shape(k), dtype=getattr(self.buffers, k).dtype, pin_memory=True)
-                         for k in self._outs}
+        dev = torch.device(device)
+        B, N, S = int(ts.n_traces), int(ts.n_tensors), int(ts.n_steps)
+        in_specs = [("trace_ptr", (B + 1,), torch.int64), ("steps", (B,), torch.int32),
+                    ("profile_ptr", (B + 1,), torch.int64), ("alloc_step", (N,), torch.int32),
+                    ("free_step", (N,), torch.int32), ("size_bytes", (N,), torch.int64)]
+        out_specs = [("profile", (S,), torch.int64), ("peak_lb", (B,), torch.int64), ("offsets", (N,), torch.int64),
+                     ("plan_peak", (B,), torch.int64), ("verdict", (B,), torch.int32),
+                     ("conflict", (2 * B,), torch.int32), ("status", (1, B), torch.int32)]
+        self.dev_in, din = _packed(in_specs, dev)
+        self.host_in_buf, self.host_in = _packed(in_specs, pin_memory=True)
+        self.dev_out, dout = _packed(out_specs, dev)
+        self.host_out_buf, self.host_out = _packed(out_specs, pin_memory=True)
+        self.stage(ts)
+        self.dev_in.copy_(self.host_in_buf)
+        self.dev_batch = DeviceBatch(din["trace_ptr"], din["steps"], din["profile_ptr"], din["alloc_step"],
+                                     din["free_step"], din["size_bytes"], B, int(ts.max_tensors),
+                                     int(ts.max_steps), N, S)
+        buf = object.__new__(PathBuffers)
+        for k in self._OUT:
+            setattr(buf, k, dout[k])
+        buf.plan_ws, buf.validate_ws = Workspace(dev), Workspace(dev)
+        buf.plan_ws.get(plan_workspace_bytes(self.dev_batch))
+        self.buffers = buf
 
     @property
     def h2d_bytes(self) -> int:
-        return sum(t.numel() * t.element_size() for t in self.host_in.values())
+        return self.host_in_buf.numel()
 
     @property
     def d2h_bytes(self) -> int:
-        return sum(t.numel() * t.element_size() for t in self.host_out.values())
+        return self.host_out_buf.numel()
 
     def stage(self, ts):
-        """Places a host batch into the pinned input buffers (host-side memcpy)."""
+        """Places a host batch into the pinned input buffer (host-side memcpy)."""
         for k in self._IN:
             self.host_in[k].numpy()[...] = getattr(ts, k)
 
@@ -379,11 +434,10 @@ class HostPath:
             self.stage(ts)
         s = self.stream or torch.cuda.current_stream()
         with torch.cuda.stream(s):
-            for k in self._IN:
-                getattr(self.dev_batch, k).copy_(self.host_in[k], non_blocking=True)
+            self.dev_in.copy_(self.host_in_buf, non_blocking=True)
             plan_and_validate(self.dev_batch, self.policy, self.buffers, stream=s)
-            for k in self._outs:
-                src = getattr(self.buffers, k)
-                self.host_out[k].copy_(src[0] if k == "status" else src, non_blocking=True)
+            self.host_out_buf.copy_(self.dev_out, non_blocking=True)
         s.synchronize()
-        return {k: v.numpy() for k, v in self.host_out.items()}
+        out = {k: v.numpy() for k, v in self.host_out.items()}
+        out["status"] = out["status"][0]
+        return out

@@ -418,3 +418,27 @@ def test_replay_on_device_slabs(cuda_lib):
     assert int(rst[1]) == oracle.EINVAL and int(ok[1]) == 0 and bool((rst[2:] == 0).all())
     r2 = rst2.cpu().numpy()
     assert (r2[:3] == 0).all() and (r2[3:][np.diff(base.cpu().numpy())[3:] > 0] == oracle.EINVAL).all()
+
+
+# ------------------------------------------------------------- end to end from host memory
+
+def test_host_path_matches_the_device_path(cuda_lib):
+    """HostPath (one pinned buffer in, one out) gives the fused call's results,
+    also for a second batch of the same shape staged into the same buffers."""
+    import paper_2203_00448_gb300 as mp
+
+    cases = ((tg.config(2).select(range(0, 4096, 8)), tg.config(2).select(range(1, 4096, 8))),
+             (tg.random_small(41, 97, 120, 200, 1 << 30),))
+    for batches in cases:
+        hp = mp.HostPath(batches[0], "cuda", "first")
+        for ts in batches:
+            ref = fused_run(ts, "first")
+            out = hp.run(ts)
+            ok = ref["st"] == 0
+            assert np.array_equal(out["status"], ref["st"])
+            for k, ptr in (("offsets", ts.trace_ptr), ("profile", ts.profile_ptr)):
+                for b in np.nonzero(ok)[0]:
+                    assert np.array_equal(out[k][ptr[b]:ptr[b + 1]], ref[k][ptr[b]:ptr[b + 1]]), (k, b)
+            for k in ("peak_lb", "plan_peak", "verdict"):
+                assert np.array_equal(out[k][ok], ref[k][ok]), k
+            assert np.array_equal(out["conflict"].reshape(-1, 2)[ok], ref["conflict"][ok])
