@@ -7,7 +7,9 @@ library.  Every function takes a ``tracegen.TraceSet`` (host numpy arrays).
 
 Passages followed: Eq. 2.1 with its pairwise ordering constraints and the
 strategy list of Sec. 2.3 (greedy_by_size, bump_allocation); Sec. 3.2 makes
-greedy_by_size the default.
+greedy_by_size the default; Sec. 6 describes greedy by breadth (operators by
+the sizes of their tensors), read here with the operator at step t using the
+tensors live at t.
 """
 from __future__ import annotations
 
@@ -61,6 +63,7 @@ def _load():
     BP = ctypes.POINTER(_Batch)
     lib.or_live_profile.argtypes = [BP, P, P, P]
     lib.or_plan_greedy_by_size.argtypes = [BP, ctypes.c_int32, P, P, P]
+    lib.or_plan_greedy_by_breadth.argtypes = [BP, ctypes.c_int32, P, P, P]
     lib.or_plan_bump.argtypes = [BP, P, P, P]
     lib.or_validate_plan.argtypes = [BP, P, P, P, P]
     lib.or_peak.argtypes = [BP, P, P, P]
@@ -105,6 +108,18 @@ def plan_greedy_by_size(ts, policy: int = FIT_FIRST):
     peak = _out(ts.n_traces, np.int64)
     st = _out(ts.n_traces, np.int32)
     lib.or_plan_greedy_by_size(ref, int(policy), off.ctypes.data, peak.ctypes.data, st.ctypes.data)
+    return off, peak, st
+
+
+def plan_greedy_by_breadth(ts, policy: int = FIT_FIRST):
+    """Greedy by breadth (operator at step t = the tensors live at t): returns
+    (offsets int64[N], plan_peak int64[B], status int32[B])."""
+    lib, keep = _load(), []
+    ref, _b = _batch(ts, keep)
+    off = _out(ts.n_tensors, np.int64)
+    peak = _out(ts.n_traces, np.int64)
+    st = _out(ts.n_traces, np.int32)
+    lib.or_plan_greedy_by_breadth(ref, int(policy), off.ctypes.data, peak.ctypes.data, st.ctypes.data)
     return off, peak, st
 
 

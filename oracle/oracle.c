@@ -151,6 +151,35 @@ static int64_t fit_in_gaps(int32_t policy, int64_t size, const int32_t *nb, int3
     return prev;
 }
 
+/* Places the tensors of one trace in the given order: each at the first or
+ * the smallest gap among the already placed, lifetime-overlapping tensors
+ * (the placement rule of greedy_by_size); returns the plan's peak. */
+static int64_t place_in_order(int32_t policy, int32_t n, const int32_t *order, const int32_t *a,
+                              const int32_t *f, const int64_t *s, int64_t *off)
+{
+    int32_t *placed = (int32_t *)malloc(sizeof(int32_t) * (size_t)(n ? n : 1));
+    int32_t *nb = (int32_t *)malloc(sizeof(int32_t) * (size_t)(n ? n : 1));
+    int32_t n_placed = 0;
+    for (int32_t r = 0; r < n; ++r) {
+        int32_t i = order[r];
+        int32_t n_nb = 0;
+        for (int32_t k = 0; k < n_placed; ++k) {
+            int32_t j = placed[k];
+            if (lifetimes_overlap(a[i], f[i], a[j], f[j])) nb[n_nb++] = j;
+        }
+        g_off = off;
+        qsort(nb, (size_t)n_nb, sizeof(int32_t), cmp_offset);
+        off[i] = fit_in_gaps(policy, s[i], nb, n_nb, off, s);
+        placed[n_placed++] = i;
+    }
+    int64_t peak = 0;
+    for (int32_t i = 0; i < n; ++i)
+        if (off[i] + s[i] > peak) peak = off[i] + s[i];
+    free(placed);
+    free(nb);
+    return peak;
+}
+
 OR_EXPORT int or_plan_greedy_by_size(const or_batch *B, int32_t policy, int64_t *offsets,
                                      int64_t *plan_peak, int32_t *trace_status)
 {
@@ -169,32 +198,76 @@ OR_EXPORT int or_plan_greedy_by_size(const or_batch *B, int32_t policy, int64_t 
             continue;
         }
         int32_t *order = (int32_t *)malloc(sizeof(int32_t) * (size_t)(n ? n : 1));
-        int32_t *placed = (int32_t *)malloc(sizeof(int32_t) * (size_t)(n ? n : 1));
-        int32_t *nb = (int32_t *)malloc(sizeof(int32_t) * (size_t)(n ? n : 1));
         for (int32_t i = 0; i < n; ++i) order[i] = i;
         g_a = a;
         g_s = s;
         qsort(order, (size_t)n, sizeof(int32_t), cmp_priority);
-        int32_t n_placed = 0;
-        for (int32_t r = 0; r < n; ++r) {
-            int32_t i = order[r];
-            int32_t n_nb = 0;
-            for (int32_t k = 0; k < n_placed; ++k) {
-                int32_t j = placed[k];
-                if (lifetimes_overlap(a[i], f[i], a[j], f[j])) nb[n_nb++] = j;
-            }
-            g_off = off;
-            qsort(nb, (size_t)n_nb, sizeof(int32_t), cmp_offset);
-            off[i] = fit_in_gaps(policy, s[i], nb, n_nb, off, s);
-            placed[n_placed++] = i;
-        }
-        int64_t peak = 0;
-        for (int32_t i = 0; i < n; ++i)
-            if (off[i] + s[i] > peak) peak = off[i] + s[i];
-        plan_peak[b] = peak;
+        plan_peak[b] = place_in_order(policy, n, order, a, f, s, off);
         free(order);
-        free(placed);
-        free(nb);
+    }
+    return 0;
+}
+
+/* ------------------------------------------------------ greedy by breadth */
+
+static const int64_t *g_m;  /* per tensor: the largest live bytes over its lifetime */
+static const int32_t *g_t;  /* per tensor: the first step at which that is reached */
+
+/* Breadth order: the widest operator first (earlier step on ties), then the
+ * greedy_by_size priority inside an operator. */
+static int cmp_breadth(const void *x, const void *y)
+{
+    int32_t i = *(const int32_t *)x, j = *(const int32_t *)y;
+    if (g_m[i] != g_m[j]) return g_m[i] > g_m[j] ? -1 : 1;
+    if (g_t[i] != g_t[j]) return g_t[i] < g_t[j] ? -1 : 1;
+    return cmp_priority(x, y);
+}
+
+OR_EXPORT int or_plan_greedy_by_breadth(const or_batch *B, int32_t policy, int64_t *offsets,
+                                        int64_t *plan_peak, int32_t *trace_status)
+{
+    for (int32_t b = 0; b < B->n_traces; ++b) {
+        int32_t st = trace_check(B, b, NULL, 0);
+        trace_status[b] = st;
+        int64_t lo = B->trace_ptr[b];
+        int32_t n = st == OR_EINVAL && (lo < 0 || B->trace_ptr[b + 1] < lo)
+                        ? 0 : (int32_t)(B->trace_ptr[b + 1] - lo);
+        const int32_t *a = B->alloc_step + lo, *f = B->free_step + lo;
+        const int64_t *s = B->size_bytes + lo;
+        int64_t *off = offsets + lo;
+        if (st != OR_OK) {
+            for (int32_t i = 0; i < n; ++i) off[i] = 0;
+            plan_peak[b] = 0;
+            continue;
+        }
+        int32_t T = B->steps[b];
+        /* operator t's breadth: the bytes of the tensors live at t */
+        int64_t *breadth = (int64_t *)calloc((size_t)(T > 0 ? T : 1), sizeof(int64_t));
+        for (int32_t i = 0; i < n; ++i)
+            for (int32_t t = a[i]; t < f[i]; ++t) breadth[t] += s[i];
+        const size_t cap = (size_t)(n > 0 ? n : 1);
+        int64_t *m = (int64_t *)malloc(sizeof(int64_t) * cap);
+        int32_t *tm = (int32_t *)malloc(sizeof(int32_t) * cap);
+        int32_t *order = (int32_t *)malloc(sizeof(int32_t) * cap);
+        for (int32_t i = 0; i < n; ++i) {
+            m[i] = -1;
+            for (int32_t t = a[i]; t < f[i]; ++t)
+                if (breadth[t] > m[i]) {
+                    m[i] = breadth[t];
+                    tm[i] = t;
+                }
+            order[i] = i;
+        }
+        g_a = a;
+        g_s = s;
+        g_m = m;
+        g_t = tm;
+        qsort(order, (size_t)n, sizeof(int32_t), cmp_breadth);
+        plan_peak[b] = place_in_order(policy, n, order, a, f, s, off);
+        free(breadth);
+        free(m);
+        free(tm);
+        free(order);
     }
     return 0;
 }

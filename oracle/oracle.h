@@ -45,6 +45,16 @@ int or_live_profile(const or_batch *b, int64_t *profile, int64_t *peak_lb, int32
 int or_plan_greedy_by_size(const or_batch *b, int32_t policy, int64_t *offsets, int64_t *plan_peak,
                            int32_t *trace_status);
 
+/* Greedy by breadth (the strategy of Pisarchyk et al. discussed in Sec. 6),
+ * read for traces without operator records: the operator at step t uses the
+ * tensors live at t, so its breadth is the live bytes at t.  Operators are
+ * taken by breadth descending (earlier step on ties), each taking its not yet
+ * placed tensors by the greedy_by_size priority; so a tensor's place in the
+ * order is the widest operator over its lifetime, then size desc, alloc asc,
+ * id asc.  Placement as greedy_by_size with the given policy. */
+int or_plan_greedy_by_breadth(const or_batch *b, int32_t policy, int64_t *offsets, int64_t *plan_peak,
+                              int32_t *trace_status);
+
 /* Pairwise constraints of Eq. 2.1: verdict 1 iff no two lifetime-overlapping
  * tensors have intersecting [offset, offset + size); conflict[2b], [2b+1] is
  * the lexicographically smallest violating (i, j), i < j, local ids, or -1. */

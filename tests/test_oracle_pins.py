@@ -283,3 +283,49 @@ def test_offset_status_codes():
     assert st.tolist() == [2]
     pk, st = oracle.peak(ts, np.array([0, 100]))
     assert st.tolist() == [0] and pk.tolist() == [108]
+
+
+# ------------------------------------------------------------- greedy by breadth
+
+def test_breadth_hand_case_orders_by_the_widest_operator():
+    """T = 2.  x: 5 bytes over [0, 2); six tensors of 4 bytes over [0, 1);
+    y: 20 bytes over [1, 2).  Operator 0 holds x and the six (29 bytes),
+    operator 1 holds x and y (25): operator 0 goes first, x (its largest) at
+    0 and the six stacked above it (5, 9, ..., 25); then y, overlapping only
+    x, at 5.  greedy_by_size instead takes y first (0), x above it (20), and
+    the six around x (0, 4, 8, 12, 16, 25)."""
+    tensors = [(0, 2, 5)] + [(0, 1, 4)] * 6 + [(1, 2, 20)]
+    ts = tg.from_tuples([(2, tensors)])
+    off, pk, st = oracle.plan_greedy_by_breadth(ts, oracle.FIT_FIRST)
+    assert st[0] == 0 and pk[0] == 29
+    assert list(off) == [0, 5, 9, 13, 17, 21, 25, 5]
+    off_s, pk_s, _ = oracle.plan_greedy_by_size(ts, oracle.FIT_FIRST)
+    assert list(off_s) == [20, 0, 4, 8, 12, 16, 25, 0] and pk_s[0] == 29
+
+
+def test_breadth_equals_size_when_every_tensor_spans_the_widest_step():
+    # every lifetime contains step 3, the widest one: one operator, size order
+    rng = np.random.default_rng(11)
+    for _ in range(20):
+        n = int(rng.integers(1, 12))
+        a = rng.integers(0, 4, n)
+        f = rng.integers(4, 8, n)
+        s = rng.integers(1, 100, n)
+        ts = tg.from_tuples([(8, list(zip(a, f, s)))])
+        for pol in (oracle.FIT_FIRST, oracle.FIT_BEST):
+            assert np.array_equal(oracle.plan_greedy_by_breadth(ts, pol)[0], oracle.plan_greedy_by_size(ts, pol)[0])
+
+
+def test_breadth_plans_are_valid_and_bounded():
+    ts = tg.random_small(13, 40, 9, 12, 1 << 10)
+    for pol in (oracle.FIT_FIRST, oracle.FIT_BEST):
+        off, pk, st = oracle.plan_greedy_by_breadth(ts, pol)
+        v, _, vst = oracle.validate_plan(ts, off)
+        _, lb, _ = oracle.live_profile(ts)
+        ok = st == 0
+        assert (v[ok] == 1).all() and (vst[ok] == 0).all()
+        assert (lb[ok] <= pk[ok]).all()
+        for b in np.nonzero(ok)[0]:
+            T, a, f, s = ts.trace(b)
+            if len(a) <= 7:
+                assert oracle.bruteforce_opt(a, f, s)[0] <= pk[b]
