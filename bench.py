@@ -67,7 +67,7 @@ def algorithmic_bytes(kernel: str, n_tensors: int, n_traces: int, n_steps: int) 
         return 24 * n_tensors + (12 + 16) * n_traces
     if kernel == FUSED:
         return 24 * n_tensors + 8 * n_steps + (20 + 32) * n_traces
-    if kernel == "plan_bump":
+    if kernel in ("plan_bump", "plan_greedy_by_breadth"):
         return 24 * n_tensors + (12 + 12) * n_traces
     raise KeyError(kernel)
 
@@ -405,6 +405,27 @@ def run_gpu(args):
             return 1
         bump_ms = sum(ev[0].elapsed_time(ev[1]) for ev in bump_events) / len(bump_events)
         next_rows = {"plan_bump": {"ms": bump_ms}}
+        # greedy by breadth on the same batch, and its plan peaks against greedy_by_size's
+        br_off = torch.empty_like(buf.offsets)
+        br_pk = torch.empty_like(buf.plan_peak)
+        br_st = torch.empty_like(buf.status[0])
+        bws = mp.Workspace(dev)
+        mp.plan_greedy_by_breadth(db, args.policy, br_off, br_pk, br_st, workspace=bws, stream=stream)
+        br_events = [mk(2) for _ in range(3)]
+        for ev in br_events:
+            flush.zero_()
+            ev[0].record(stream)
+            mp.plan_greedy_by_breadth(db, args.policy, br_off, br_pk, br_st, workspace=bws, stream=stream)
+            ev[1].record(stream)
+        torch.cuda.synchronize()
+        if not bool((br_st == 0).all()):
+            print(json.dumps({"error": "plan_greedy_by_breadth reported a failed trace", "rank": rank}))
+            return 1
+        pk_ratio = br_pk.double() / buf.plan_peak.double()
+        next_rows["plan_greedy_by_breadth"] = {
+            "ms": sum(ev[0].elapsed_time(ev[1]) for ev in br_events) / len(br_events),
+            "peak_over_greedy_by_size": {"mean": float(pk_ratio.mean()), "min": float(pk_ratio.min()),
+                                         "max": float(pk_ratio.max())}}
         # The exact optimum on small traces (the generator of the bench
         # workload, 9 tensors over 6 steps, so that lifetimes overlap) and the
         # gap of the greedy plan to it.
@@ -462,7 +483,7 @@ def run_gpu(args):
         kern[name] = {"ms": per_kernel[j], "algorithmic_bytes": nbytes, "achieved_gbs": gbs, "frac": gbs / peak}
     if next_rows is not None:
         for name, row in next_rows.items():
-            if name != "plan_bump":
+            if name not in ("plan_bump", "plan_greedy_by_breadth"):
                 continue  # the exhaustive search is bound by its n! placements, not by memory
             nbytes = algorithmic_bytes(name, ts.n_tensors, ts.n_traces, n_steps)
             gbs = nbytes / (row["ms"] * 1e-3) / 1e9

@@ -207,6 +207,25 @@ size_t mp_bump_workspace_bytes(const mp_batch *batch);
 mp_status mp_plan_bump(const mp_batch *batch, int64_t *offsets, int64_t *plan_peak, int32_t *trace_status,
                        void *workspace, size_t workspace_bytes, void *stream);
 
+/* Bytes of device workspace mp_plan_greedy_by_breadth needs for this batch. */
+size_t mp_breadth_workspace_bytes(const mp_batch *batch);
+
+/* Greedy by breadth, the strategy of Pisarchyk et al. discussed in Sec. 6:
+ * operators in order of breadth (the sizes of the tensors they use)
+ * descending, each assigning offsets to its tensors not yet placed, largest
+ * first, with greedy_by_size's gap search (policy as for
+ * mp_plan_greedy_by_size).  Traces carry no operator records, so the operator
+ * at step t is read as using the tensors live at t (breadth = live bytes at
+ * t; ties: the earlier step first): a tensor is placed with the widest
+ * operator over its lifetime.
+ * offsets, plan_peak, trace_status as for mp_plan_greedy_by_size (a failed
+ * trace gets plan_peak 0).  workspace: at least
+ * mp_breadth_workspace_bytes(batch) bytes, rules as for
+ * mp_plan_greedy_by_size. */
+mp_status mp_plan_greedy_by_breadth(const mp_batch *batch, mp_fit_policy policy, int64_t *offsets,
+                                    int64_t *plan_peak, int32_t *trace_status, void *workspace,
+                                    size_t workspace_bytes, void *stream);
+
 /* Traces of at most this many tensors are searched exhaustively by
  * mp_plan_optimal. */
 #define MP_OPTIMAL_MAX_TENSORS 10

@@ -27,6 +27,8 @@ EXPORTS = (
     "mp_plan_bump",
     "mp_optimal_workspace_bytes",
     "mp_plan_optimal",
+    "mp_breadth_workspace_bytes",
+    "mp_plan_greedy_by_breadth",
     "mp_slab_layout",
     "mp_replay_workspace_bytes",
     "mp_replay_plan",
@@ -98,6 +100,10 @@ def load(path: str = LIB_PATH):
     lib.mp_optimal_workspace_bytes.restype = sz
     lib.mp_plan_optimal.argtypes = [BP, P, P, P, P, sz, P]
     lib.mp_plan_optimal.restype = i32
+    lib.mp_breadth_workspace_bytes.argtypes = [BP]
+    lib.mp_breadth_workspace_bytes.restype = sz
+    lib.mp_plan_greedy_by_breadth.argtypes = [BP, i32, P, P, P, P, sz, P]
+    lib.mp_plan_greedy_by_breadth.restype = i32
     lib.mp_slab_layout.argtypes = [i32, P, P, P]
     lib.mp_slab_layout.restype = i32
     lib.mp_replay_workspace_bytes.argtypes = [BP]

@@ -233,6 +233,22 @@ def plan_bump(batch: DeviceBatch, offsets=None, plan_peak=None, status=None, wor
     return offsets, plan_peak, status
 
 
+def plan_greedy_by_breadth(batch: DeviceBatch, policy="first", offsets=None, plan_peak=None, status=None,
+                           workspace: "Workspace | None" = None, stream=None):
+    """Greedy by breadth (Sec. 6; the operator at step t uses the tensors live
+    at t).  Returns (offsets, plan_peak, status)."""
+    lib, dev = _lib.load(), batch.device
+    offsets = _empty(batch.n_tensors, torch.int64, dev) if offsets is None else offsets
+    plan_peak = _empty(batch.n_traces, torch.int64, dev) if plan_peak is None else plan_peak
+    status = _empty(batch.n_traces, torch.int32, dev) if status is None else status
+    s = batch.struct()
+    wptr, wbytes = _workspace(workspace, dev).get(int(lib.mp_breadth_workspace_bytes(ctypes.byref(s))))
+    _check("mp_plan_greedy_by_breadth",
+           lib.mp_plan_greedy_by_breadth(ctypes.byref(s), _policy(policy), _ptr(offsets), _ptr(plan_peak),
+                                         _ptr(status), wptr, wbytes, _stream_ptr(stream)))
+    return offsets, plan_peak, status
+
+
 def plan_optimal(batch: DeviceBatch, offsets=None, opt_peak=None, status=None, workspace: "Workspace | None" = None,
                  stream=None):
     """The exact optimum of Eq. 2.1 for traces of at most 10 tensors (exhaustive

@@ -255,6 +255,26 @@ __attribute__((visibility("default"))) mp_status mp_replay_plan(const mp_batch* 
                                        first_bad, trace_status, workspace, static_cast<cudaStream_t>(stream)));
 }
 
+__attribute__((visibility("default"))) size_t mp_breadth_workspace_bytes(const mp_batch* batch) {
+    if (check_batch(batch, false) != MP_OK) return 0;
+    return mp::breadth_workspace_bytes(*batch);
+}
+
+__attribute__((visibility("default"))) mp_status mp_plan_greedy_by_breadth(
+    const mp_batch* batch, mp_fit_policy policy, int64_t* offsets, int64_t* plan_peak, int32_t* trace_status,
+    void* workspace, size_t workspace_bytes, void* stream) {
+    mp_status st = check_batch(batch, false);
+    if (st != MP_OK) return st;
+    if (policy != MP_FIT_FIRST && policy != MP_FIT_BEST) return MP_EINVAL;
+    if (!array_ok(offsets, batch->n_tensors) || !array_ok(plan_peak, batch->n_traces) ||
+        !array_ok(trace_status, batch->n_traces))
+        return MP_EINVAL;
+    st = check_workspace(mp::breadth_workspace_bytes(*batch), workspace, workspace_bytes);
+    if (st != MP_OK) return st;
+    return from_cuda(mp::launch_breadth(*batch, policy, offsets, plan_peak, trace_status, workspace,
+                                        static_cast<cudaStream_t>(stream)));
+}
+
 __attribute__((visibility("default"))) mp_status mp_peak(const mp_batch* batch, const int64_t* offsets,
                                                          int64_t* plan_peak, int32_t* trace_status,
                                                          void* stream) {

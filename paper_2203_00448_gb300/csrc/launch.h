@@ -16,6 +16,7 @@ constexpr int kPeakThreads = 256;
 constexpr int kBumpThreads = 128;
 constexpr int kOptThreads = 128;
 constexpr int kReplayThreads = 256;
+constexpr int kBreadthThreads = 128;
 constexpr int kPlanThreadsSmem = 128;    // one CTA per trace, data in shared memory
 constexpr int kPlanThreadsGlobal = 1024; // one CTA per trace, data in the workspace
 
@@ -57,6 +58,10 @@ cudaError_t launch_slab_layout(int32_t n_traces, const int64_t* plan_peak, int64
 cudaError_t launch_replay(const mp_batch& bt, const int64_t* offsets, const int64_t* slab_base, unsigned char* slab,
                           int64_t slab_bytes, int32_t* ok, int32_t* first_bad, int32_t* status, void* workspace,
                           cudaStream_t stream);
+
+size_t breadth_workspace_bytes(const mp_batch& bt);
+cudaError_t launch_breadth(const mp_batch& bt, int32_t policy, int64_t* offsets, int64_t* plan_peak, int32_t* status,
+                           void* workspace, cudaStream_t stream);
 
 cudaError_t launch_peak(const mp_batch& bt, const int64_t* offsets, int64_t* plan_peak, int32_t* status,
                         cudaStream_t stream);

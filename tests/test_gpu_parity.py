@@ -442,3 +442,25 @@ def test_host_path_matches_the_device_path(cuda_lib):
             for k in ("peak_lb", "plan_peak", "verdict"):
                 assert np.array_equal(out[k][ok], ref[k][ok]), k
             assert np.array_equal(out["conflict"].reshape(-1, 2)[ok], ref["conflict"][ok])
+
+
+# ------------------------------------------------------------- greedy by breadth
+
+@pytest.mark.parametrize("name,pol", POLICIES)
+def test_breadth_parity(cuda_lib, name, pol):
+    import paper_2203_00448_gb300 as mp
+
+    hand = tg.from_tuples([(2, [(0, 2, 5)] + [(0, 1, 4)] * 6 + [(1, 2, 20)])])
+    for ts in (tg.config(0), tg.config(1), tg.config(2).select(range(0, 4096, 16)), tg.config(3), hand,
+               tg.random_small(17, 200, 100, 150, 1 << 24),
+               tg.from_tuples([(4, [(-1, 2, 8)]), (4, [(0, 1, 2 ** 62), (0, 2, 2 ** 62)]), (0, []), (5, [])])):
+        db = mp.DeviceBatch.from_host(ts, "cuda")
+        off, pk, st = mp.plan_greedy_by_breadth(db, name)
+        torch.cuda.synchronize()
+        o_off, o_pk, o_st = oracle.plan_greedy_by_breadth(ts, pol)
+        st, pk, off = st.cpu().numpy(), pk.cpu().numpy(), off.cpu().numpy()
+        assert np.array_equal(st, o_st), ts.name
+        assert np.array_equal(pk, o_pk), ts.name
+        for b in np.nonzero(o_st == 0)[0]:
+            lo, hi = ts.trace_ptr[b], ts.trace_ptr[b + 1]
+            assert np.array_equal(off[lo:hi], o_off[lo:hi]), (ts.name, b)
