@@ -98,3 +98,29 @@ def test_product_path_never_touches_the_oracle():
             if fn.endswith((".py", ".cu", ".cuh", ".h")):
                 src = open(os.path.join(dirpath, fn)).read()
                 assert not re.search(r"\bimport\s+oracle\b|\bfrom\s+oracle\b|liboracle|oracle\.h", src), fn
+
+
+def test_host_argument_errors_of_the_other_strategies(lib):
+    """The entry points beyond the hot path reject bad host arguments before
+    anything is enqueued (fake device addresses are never dereferenced)."""
+    P = 0x10000
+    EINVAL, ENOMEM = _lib.EINVAL, _lib.ENOMEM
+    b = _batch()
+    assert lib.mp_plan_bump(None, P, P, P, None, 0, None) == EINVAL
+    assert lib.mp_plan_bump(ctypes.byref(b), None, P, P, None, 0, None) == EINVAL
+    assert lib.mp_plan_bump(ctypes.byref(b), P, P + 4, P, None, 0, None) == EINVAL   # misaligned int64
+    assert lib.mp_plan_greedy_by_breadth(ctypes.byref(b), 5, P, P, P, None, 0, None) == EINVAL  # policy
+    assert lib.mp_plan_greedy_by_breadth(ctypes.byref(b), 0, P, None, P, None, 0, None) == EINVAL
+    need = lib.mp_optimal_workspace_bytes(ctypes.byref(b))
+    assert need > 0
+    assert lib.mp_plan_optimal(ctypes.byref(b), P, P, P, P, need - 1, None) == ENOMEM
+    assert lib.mp_plan_optimal(ctypes.byref(b), P, P, P, None, need, None) == EINVAL
+    assert lib.mp_slab_layout(-1, P, P, None) == EINVAL
+    assert lib.mp_slab_layout(4, None, P, None) == EINVAL
+    assert lib.mp_replay_plan(ctypes.byref(b), P, P, None, 64, P, P, P, None, 0, None) == EINVAL  # no slab
+    assert lib.mp_replay_plan(ctypes.byref(b), P, P, P, -1, P, P, P, None, 0, None) == EINVAL     # negative size
+    assert lib.mp_replay_plan(ctypes.byref(b), P, None, P, 64, P, P, P, None, 0, None) == EINVAL  # no slab bases
+    big = _batch(max_tensors=20000, max_steps=10000)
+    for fn in ("mp_bump_workspace_bytes", "mp_breadth_workspace_bytes", "mp_replay_workspace_bytes"):
+        assert getattr(lib, fn)(ctypes.byref(_batch())) == 0  # small traces: shared memory
+        assert getattr(lib, fn)(ctypes.byref(big)) > 0
