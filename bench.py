@@ -133,9 +133,10 @@ def kernel_source_digest() -> str:
     return h.hexdigest()
 
 
-def ncu_traffic(kernel: str, n_tensors: int):
-    """DRAM bytes per launch from the committed ncu capture, scaled to this
-    launch's tensor count; None if absent or if the kernels changed since."""
+def ncu_record(kernel: str, n_tensors: int, field: str = "dram_bytes"):
+    """A per-launch counter (DRAM bytes, warp instructions) from the committed
+    ncu capture, scaled to this launch's tensor count; None if absent or if the
+    kernels changed since."""
     path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
     try:
         with open(path) as f:
@@ -145,9 +146,27 @@ def ncu_traffic(kernel: str, n_tensors: int):
     if d.get("source_sha256") != kernel_source_digest():
         return None
     k = d.get("kernels", {}).get(kernel)
-    if not k:
+    if not k or field not in k:
         return None
-    return k["dram_bytes"] * n_tensors / k["n_tensors"]
+    return k[field] * n_tensors / k["n_tensors"]
+
+
+# Each SM has four schedulers that issue one warp instruction per cycle each.
+ISSUE_PER_SM_PER_CLK = 4
+
+
+def issue_roofline(warp_inst: float, seconds: float, n_sms: int, sm_mhz: float):
+    """Second roofline for the integer planner, which is issue-bound rather than
+    HBM-bound: warp instructions per second against n_sms * 4 * clock."""
+    if warp_inst is None or not sm_mhz:
+        return None
+    peak = n_sms * ISSUE_PER_SM_PER_CLK * sm_mhz * 1e6
+    achieved = warp_inst / seconds
+    return {"bound": "issue", "achieved": achieved, "peak": peak, "unit": "warp-inst/s", "frac": achieved / peak,
+            "warp_inst_per_launch": warp_inst,
+            "peak_source": f"{n_sms} SMs x {ISSUE_PER_SM_PER_CLK} warp-inst/clk x {sm_mhz:.0f} MHz (median SM clock "
+                           f"sampled during the timed steps)",
+            "inst_source": "smsp__inst_executed.sum of the committed ncu capture, scaled by tensors"}
 
 
 def gpu_id(dev) -> str:
@@ -494,7 +513,7 @@ def run_gpu(args):
             row.update({"algorithmic_bytes": nbytes, "achieved_gbs": gbs, "frac": gbs / peak})
     fused_bytes = algorithmic_bytes(FUSED, ts.n_tensors, ts.n_traces, n_steps)
     fused_gbs = fused_bytes / (step_ms * 1e-3) / 1e9
-    traffic = ncu_traffic(FUSED, ts.n_tensors)
+    traffic = ncu_record(FUSED, ts.n_tensors)
     roof = {"bound": "hbm",
             "kernel": "k_plan, fused profile + plan + validate (one mp_plan_and_validate call: the 32-bit launch "
                       "and the 64-bit launch, which returns at once on this workload)",
@@ -509,6 +528,9 @@ def run_gpu(args):
     else:
         cpu_baseline = None
     clocks = sampler.summary()
+    issue = issue_roofline(ncu_record(FUSED, ts.n_tensors, "warp_inst"), step_ms * 1e-3,
+                           torch.cuda.get_device_properties(dev).multi_processor_count,
+                           clocks["sm_mhz"] or clocks["sm_max_mhz"])
     line = {
         "metric": METRIC, "value": total_tensors / (step_ms_max * 1e-3), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms_max, "higher_is_better": True,
@@ -525,6 +547,7 @@ def run_gpu(args):
         "separate_kernels": kern,
         "next_rows": next_rows,
         "roofline": roof,
+        "issue_roofline": issue,
         "cpu_baseline": cpu_baseline,
         "e2e": e2e,
         "clocks": clocks,
