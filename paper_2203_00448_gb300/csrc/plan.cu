@@ -66,9 +66,12 @@ namespace {
 
 constexpr int32_t kThreadComp = 8;   // components up to this size: one thread
 constexpr int32_t kWarpComp = 32;    // ... up to this size: one warp (a tensor per lane); else the CTA
-constexpr int32_t kCandMax = 64;     // CTA tier: up to this many predecessors, test all candidates
 constexpr int kCached = 4;           // tensors per thread kept in registers between the two input passes
-constexpr int64_t kNone = INT64_MAX;
+constexpr int32_t kLongLife = 32;    // CTA tier: members living longer than this many steps are listed apart
+constexpr int32_t kPredBuf = 128;    // CTA tier, data in the workspace: predecessors gathered per warp
+constexpr int32_t kLongStage = 2048; // CTA tier, data in the workspace: long-lived members staged in shared memory
+constexpr long long kSpinCycles = 1ll << 31;  // a wait for another warp longer than this is a fault
+constexpr int32_t kValWide = 64;     // validation: windows longer than this get a warp each
 constexpr int32_t kDeferred = -1;    // trace status between the two launches: needs 64-bit bytes
 
 // Component size classes for the counting sort of the component list:
@@ -114,17 +117,11 @@ __host__ __device__ constexpr size_t dpadded(size_t T) {
     return T + ProfGeom<W>::kPad * ((T + ProfGeom<W>::kRun - 1) / ProfGeom<W>::kRun);
 }
 
-// A tensor in alloc-step order; in priority order for the CTA tier (with its
-// alloc-order position), which always works in 64-bit bytes.
+// A tensor in alloc-step order.
 template <typename I, typename W>
 struct ARec {
     W s;
     I a, f, id, pad;
-};
-template <typename I>
-struct SRec {
-    int64_t s, off;
-    I a, f, id, pos;
 };
 
 // Per-trace working set.  The records and the offsets (by alloc-order
@@ -132,7 +129,7 @@ struct SRec {
 // dead before the records are written.
 template <typename I, typename W>
 struct PlanLayout {
-    size_t arec, offp, dprof, bend, sb, lst, rp, total;
+    size_t arec, offp, dprof, bend, sb, wt, lst, rp, ord, cnt, que, total;
     __host__ __device__ PlanLayout(int64_t n, int64_t T, bool fused) {
         arec = 0;
         offp = arec + align16((size_t)n * sizeof(ARec<I, W>));
@@ -141,9 +138,13 @@ struct PlanLayout {
         const size_t dend = fused ? align16(dpadded<W>((size_t)T) * sizeof(W)) : 0;
         bend = main_end > dend ? main_end : dend;
         sb = bend + align16((size_t)T * 4);
-        lst = sb + align16((size_t)((n + 31) / 32) * 4);
-        rp = lst + align16((size_t)n * 4);
-        total = align_up(rp + align16((size_t)n * 2));
+        wt = sb + align16((size_t)((n + 31) / 32) * 4);
+        lst = wt + align16((size_t)((n + 31) / 32) * 8);
+        rp = lst + align16((size_t)n * 4);   // later the CTA tier's long-lived ranks (int32)
+        ord = rp + align16((size_t)n * 4);   // the CTA tier's priority order (int32)
+        cnt = ord + align16((size_t)n * 4);  // the CTA tier's predecessor counts (int32)
+        que = cnt + align16((size_t)n * 4);  // the CTA tier's ready queue (int32)
+        total = align_up(que + align16((size_t)n * 4));
     }
 };
 
@@ -400,129 +401,539 @@ __device__ __forceinline__ int64_t block_excl_max(int64_t v, int64_t* red, int64
     return r;
 }
 
-struct CtaScratch {
-    int64_t* red;  // >= 64 slots
-    int32_t* cnt;
-    unsigned long long* top;
+// Waits until another warp fills *slot (-1 until then) and returns it.
+// Gives up after kSpinCycles, or at once when another warp has given up,
+// and then sets *fail and returns -1.
+__device__ __forceinline__ int32_t wait_slot(const volatile int32_t* slot, volatile int32_t* fail) {
+    int32_t v = *slot;
+    if (v >= 0) return v;
+    const long long t0 = clock64();
+    for (;;) {
+        __nanosleep(64);
+        v = *slot;
+        if (v >= 0) return v;
+        if (*fail || clock64() - t0 > kSpinCycles) {
+            *fail = 1;
+            return -1;
+        }
+    }
+}
+
+// Position of the (n + 1)-th set bit of m (n < popc(m)).
+__device__ __forceinline__ int nth_set_bit(unsigned m, int n) {
+    int pos = 0;
+#pragma unroll
+    for (int step = 16; step > 0; step >>= 1)
+        if (__popc(m & ((1u << (pos + step)) - 1u)) <= n) pos += step;
+    return pos;
+}
+
+// A large component in the CTA tier.  Its members in priority order are
+// ord[0, c) (positions); the long-lived ones (life above kLongLife steps) are
+// at the ranks hr[0, nl), ascending.  A short-lived member x can only overlap
+// members allocated in (a_x - kLongLife, f_x) -- a window of alloc order
+// (BEND[t] = tensors allocated at or before t) -- or long-lived ones.  The
+// variant with its data in the workspace stages the first kLongStage
+// long-lived members in shared memory, by list index.
+template <typename W>
+struct LongStage {
+    W* s;
+    W* off;
+    int32_t* a;
+    int32_t* f;
+    int32_t* id;
+};
+template <typename I, typename W>
+struct Comp {
+    const ARec<I, W>* AR;
+    W* OFFP;
+    const int32_t* BEND;
+    const int32_t* ord;
+    const int32_t* hr;
+    int32_t p0, c, nl;
+    LongStage<W> st;
+    bool staged;
+
+    __device__ __forceinline__ void window(const ARec<I, W>& me, int32_t& w0, int32_t& w1) const {
+        w0 = max(p0, (int32_t)me.a >= kLongLife ? BEND[(int32_t)me.a - kLongLife] : 0);
+        w1 = min(p0 + c, BEND[(int32_t)me.f - 1]);
+    }
+    // The k-th long-lived member (record and offset; the offset once placed).
+    __device__ __forceinline__ ARec<I, W> long_rec(int32_t k, int32_t& pos) const {
+        pos = ord[hr[k]];
+        if (staged) {
+            ARec<I, W> o;
+            o.s = st.s[k];
+            o.a = (I)st.a[k];
+            o.f = (I)st.f[k];
+            o.id = (I)st.id[k];
+            return o;
+        }
+        return AR[pos];
+    }
+    __device__ __forceinline__ W long_off(int32_t k, int32_t pos) const { return staged ? st.off[k] : OFFP[pos]; }
 };
 
-// Places the priority-ordered records R[0, c) of one component with the whole
-// CTA.  bo/be: workspace buffers of at least pow2_at_least(c) entries each.
-template <typename I>
-__device__ void place_large(SRec<I>* R, int32_t c, int32_t policy, int64_t* bo, int64_t* be, const CtaScratch& sc) {
-    for (int32_t r = 0; r < c; ++r) {
-        const int64_t s = R[r].s;
-        const int32_t ai = R[r].a, fi = R[r].f;
-        if (threadIdx.x == 0) {
-            *sc.cnt = 0;
-            *sc.top = 0;
-        }
-        __syncthreads();
-        for (int32_t x = threadIdx.x; x < r; x += blockDim.x) {  // placed, lifetime-overlapping
-            if (R[x].a < fi && ai < R[x].f) {
-                const int64_t o = R[x].off, e = o + R[x].s;
-                const int32_t pos = atomicAdd(sc.cnt, 1);
-                bo[pos] = o;
-                be[pos] = e;
-                atomicMax(sc.top, (unsigned long long)e);
-            }
-        }
-        __syncthreads();
-        const int32_t P = *sc.cnt;
-        const int64_t top = (int64_t)*sc.top;
-        int64_t key = kNone, val = kNone;
-        if (P <= kCandMax) {
-            for (int32_t k = threadIdx.x; k <= P; k += blockDim.x) {
-                const int64_t cand = k == 0 ? 0 : be[k - 1];
-                if (policy == MP_FIT_FIRST) {
-                    bool ok = true;
-                    for (int32_t x = 0; x < P && ok; ++x) ok = !(bo[x] < cand + s && cand < be[x]);
-                    if (ok && cand < key) key = val = cand;
-                } else if (cand < top) {
-                    int64_t next = INT64_MAX;
-                    bool covered = false;
-                    for (int32_t x = 0; x < P && !covered; ++x) {
-                        covered = bo[x] <= cand && cand < be[x];
-                        if (bo[x] >= cand && bo[x] < next) next = bo[x];
-                    }
-                    const int64_t gl = next - cand;
-                    if (!covered && gl >= s && (gl < key || (gl == key && cand < val))) {
-                        key = gl;
-                        val = cand;
-                    }
-                }
-            }
-            block_min_pair(key, val, sc.red);
-        } else if (policy == MP_FIT_FIRST) {
-            int64_t o = 0;
-            for (;;) {
-                int64_t next = o;
-                for (int32_t x = threadIdx.x; x < P; x += blockDim.x)
-                    if (bo[x] < o + s && o < be[x] && be[x] > next) next = be[x];
-                next = block_max_i64(next, sc.red);
-                if (next == o) break;
-                o = next;
-            }
-            key = val = o;
-        } else {
-            // Sort predecessors by offset, then gap_k = off_(k) - max end of those before k.
-            const int32_t plen = (int32_t)pow2_at_least(P);
-            for (int32_t x = P + threadIdx.x; x < plen; x += blockDim.x) {
-                bo[x] = INT64_MAX;
-                be[x] = INT64_MAX;
-            }
-            __syncthreads();
-            for (int32_t k = 2; k <= plen; k <<= 1) {
-                for (int32_t j = k >> 1; j > 0; j >>= 1) {
-                    for (int32_t t = threadIdx.x; t < (plen >> 1); t += blockDim.x) {
-                        const int32_t lo = 2 * t - (t & (j - 1)), hi = lo + j;
-                        const bool up = (lo & k) == 0;
-                        const int64_t xo = bo[lo], yo = bo[hi];
-                        if (up ? yo < xo : xo < yo) {
-                            const int64_t xe = be[lo];
-                            bo[lo] = yo;
-                            bo[hi] = xo;
-                            be[lo] = be[hi];
-                            be[hi] = xe;
-                        }
-                    }
-                    __syncthreads();
-                }
-            }
-            const int32_t chunk = (P + blockDim.x - 1) / blockDim.x;
-            const int32_t k0 = min(P, (int32_t)threadIdx.x * chunk), k1 = min(P, k0 + chunk);
-            int64_t local = 0;
-            for (int32_t k = k0; k < k1; ++k) local = be[k] > local ? be[k] : local;
-            int64_t total;
-            int64_t prev = block_excl_max(local, sc.red, &total);
-            for (int32_t k = k0; k < k1; ++k) {
-                const int64_t gl = bo[k] - prev;
-                if (gl >= s && (gl < key || (gl == key && prev < val))) {
-                    key = gl;
-                    val = prev;
-                }
-                prev = be[k] > prev ? be[k] : prev;
-            }
-            block_min_pair(key, val, sc.red);
-        }
-        if (threadIdx.x == 0) R[r].off = (policy == MP_FIT_FIRST) ? key : (key == kNone ? top : val);
-        __syncthreads();
+// Shared memory of the workspace variant: the long-lived stage, then a
+// scratch area -- one predecessor buffer of kPredBuf (offset, end) pairs per
+// warp while short-lived members are placed, the predecessors of a
+// long-lived member while it is placed.
+constexpr size_t kScratchBytes = 128 * 1024;
+template <typename W>
+__host__ __device__ constexpr size_t flow_smem_bytes() {
+    return (size_t)kLongStage * (2 * sizeof(W) + 12) + kScratchBytes;
+}
+template <typename W>
+__device__ __forceinline__ LongStage<W> long_stage(unsigned char* smem, W** scratch) {
+    LongStage<W> st;
+    W* w = reinterpret_cast<W*>(smem);
+    st.s = w;
+    st.off = w + kLongStage;
+    *scratch = w + 2 * kLongStage;
+    int32_t* i = reinterpret_cast<int32_t*>(reinterpret_cast<unsigned char*>(*scratch) + kScratchBytes);
+    st.a = i;
+    st.f = i + kLongStage;
+    st.id = i + 2 * kLongStage;
+    return st;
+}
+
+// Places the short-lived members of ranks [r0, r1) of a component (a run
+// between two long-lived members; every lower rank is placed) with every
+// warp of the CTA, in dependency order.  Each member counts its predecessors
+// inside the run (the members that come first in priority and overlap its
+// lifetime); members with none are queued.  A warp takes the next queued
+// member, places it -- its offset depends on its predecessors' alone, so it
+// is the sequential definition's -- publishes the offset, and decrements
+// its successors inside the run, queuing those that reach zero.  Every
+// member is queued exactly once, and the lowest unplaced rank is always
+// ready, so the queue always fills.  Predecessors are gathered once: into a
+// register per lane when there are at most 32, else into the warp's buffer
+// pb (kPredBuf pairs) when there is one, else every pass of the gap search
+// visits the candidates again.  Returns the largest end placed (lane 0).
+template <typename I, typename W>
+__device__ W place_run(const Comp<I, W>& cp, int32_t r0, int32_t r1, int32_t nl_placed, int32_t* CNT,
+                       int32_t* QUE, W* pb, int32_t policy, int32_t* head, int32_t* tail, volatile int32_t* fail) {
+    const unsigned full = 0xffffffffu;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+    const unsigned lt_mask = (1u << lane) - 1u;
+    const int32_t len = r1 - r0;
+    volatile W* voff = cp.OFFP;
+    volatile int32_t* vque = QUE;
+    for (int32_t i = threadIdx.x; i < len; i += blockDim.x) QUE[i] = -1;
+    if (threadIdx.x == 0) {
+        *head = 0;
+        *tail = 0;
     }
+    __syncthreads();
+    const ARec<I, W> R0 = cp.AR[cp.ord[r0]];
+    const bool last = r1 == cp.c;
+    const ARec<I, W> R1 = cp.AR[cp.ord[last ? r0 : r1]];
+    auto is_short = [](const ARec<I, W>& o) { return (int32_t)o.f - (int32_t)o.a <= kLongLife; };
+    auto overlaps = [](const ARec<I, W>& o, const ARec<I, W>& me) {
+        return (int32_t)o.a < (int32_t)me.f && (int32_t)me.a < (int32_t)o.f;
+    };
+    auto push = [&](int32_t x) {
+        const int32_t at = atomicAdd(tail, 1);
+        vque[at] = x;
+    };
+
+    // predecessors inside the run, a warp per member
+    for (int32_t r = r0 + warp; r < r1; r += nwarps) {
+        const int32_t x = cp.ord[r];
+        const ARec<I, W> me = cp.AR[x];
+        int32_t w0, w1;
+        cp.window(me, w0, w1);
+        int32_t cnt = 0;
+        for (int32_t q0 = w0; q0 < w1; q0 += 32) {
+            const int32_t q = q0 + lane;
+            bool hit = false;
+            if (q < w1 && q != x) {
+                const ARec<I, W> o = cp.AR[q];
+                hit = is_short(o) && overlaps(o, me) && precedes(o, me) && !precedes(o, R0);
+            }
+            cnt += __popc(__ballot_sync(full, hit));
+        }
+        if (lane == 0) {
+            CNT[x] = cnt;
+            if (cnt == 0) push(x);
+        }
+    }
+    __syncthreads();
+
+    W mx = 0;
+    for (;;) {
+        int32_t idx = 0;
+        if (lane == 0) idx = atomicAdd(head, 1);
+        idx = __shfl_sync(full, idx, 0);
+        if (idx >= len) break;
+        int32_t x = 0;
+        if (lane == 0) x = wait_slot(vque + idx, fail);
+        x = __shfl_sync(full, x, 0);
+        if (x < 0) break;
+        __threadfence_block();  // the predecessors' offsets after the queue entry
+        const ARec<I, W> me = cp.AR[x];
+        const W s = me.s;
+        int32_t w0, w1;
+        cp.window(me, w0, w1);
+        // scan(fn): fn(is_pred, off, end) on every lane for each candidate, in
+        // warp-uniform rounds
+        auto scan = [&](auto&& fn) {
+            for (int32_t q0 = w0; q0 < w1; q0 += 32) {
+                const int32_t q = q0 + lane;
+                bool hit = false;
+                W po = 0, pe = 0;
+                if (q < w1 && q != x) {
+                    const ARec<I, W> o = cp.AR[q];
+                    if (is_short(o) && overlaps(o, me) && precedes(o, me)) {
+                        hit = true;
+                        po = voff[q];
+                        pe = po + o.s;
+                    }
+                }
+                fn(hit, po, pe);
+            }
+            for (int32_t k0 = 0; k0 < nl_placed; k0 += 32) {
+                const int32_t k = k0 + lane;
+                bool hit = false;
+                W po = 0, pe = 0;
+                if (k < nl_placed) {
+                    int32_t q;
+                    const ARec<I, W> o = cp.long_rec(k, q);
+                    if (overlaps(o, me)) {  // placed before this run: it precedes
+                        hit = true;
+                        po = cp.long_off(k, q);
+                        pe = po + o.s;
+                    }
+                }
+                fn(hit, po, pe);
+            }
+        };
+        W rpo = 0, rpe = 0;  // register mode: lane l holds predecessor l
+        int32_t np = 0;
+        scan([&](bool hit, W po, W pe) {
+            const unsigned bal = __ballot_sync(full, hit);
+            if (bal == 0) return;
+            const int32_t cnt = __popc(bal), rel = lane - np;
+            const bool mine = rel >= 0 && rel < cnt;
+            const int src = mine ? nth_set_bit(bal, rel) : lane;
+            const W so = __shfl_sync(full, po, src), se = __shfl_sync(full, pe, src);
+            if (mine) {
+                rpo = so;
+                rpe = se;
+            }
+            if (pb != nullptr) {
+                const int32_t at = np + __popc(bal & lt_mask);
+                if (hit && at < kPredBuf) {
+                    pb[2 * at] = po;
+                    pb[2 * at + 1] = pe;
+                }
+            }
+            np += cnt;
+        });
+        __syncwarp();
+        const int mode = np <= 32 ? 0 : (pb != nullptr && np <= kPredBuf ? 1 : 2);
+        // each(fn): fn(off, end) for every predecessor held by this lane
+        auto each = [&](auto&& fn) {
+            if (mode == 0) {
+                if (lane < np) fn(rpo, rpe);
+            } else if (mode == 1) {
+                for (int32_t k = lane; k < np; k += 32) fn(pb[2 * k], pb[2 * k + 1]);
+            } else {
+                scan([&](bool hit, W po, W pe) {
+                    if (hit) fn(po, pe);
+                });
+            }
+        };
+        W o = 0;
+        if (policy == MP_FIT_FIRST) {
+            for (;;) {
+                W hit = 0;
+                each([&](W po, W pe) {
+                    if (po < o + s && o < pe && pe > hit) hit = pe;
+                });
+                hit = warp_max_w(hit);
+                if (hit <= o) break;
+                o = hit;
+            }
+        } else {
+            W top = 0;
+            each([&](W, W pe) { top = pe > top ? pe : top; });
+            top = warp_max_w(top);
+            W cc = 0, best_len = w_none<W>();
+            o = top;
+            while (cc < top) {
+                for (;;) {  // move cc off any predecessor that covers it
+                    W cov = 0;
+                    each([&](W po, W pe) {
+                        if (po <= cc && cc < pe && pe > cov) cov = pe;
+                    });
+                    cov = warp_max_w(cov);
+                    if (cov <= cc) break;
+                    cc = cov;
+                }
+                if (cc >= top) break;
+                W ns = w_none<W>();
+                each([&](W po, W) {
+                    if (po > cc && po < ns) ns = po;
+                });
+                ns = warp_min_w(ns);
+                const W len2 = ns - cc;
+                if (len2 >= s && len2 < best_len) {
+                    best_len = len2;
+                    o = cc;
+                }
+                cc = ns;
+            }
+        }
+        if (lane == 0) {
+            voff[x] = o;
+            __threadfence_block();  // the offset before any successor can be queued
+            mx = o + s > mx ? o + s : mx;
+        }
+        __syncwarp();
+        // successors inside the run
+        for (int32_t q0 = w0; q0 < w1; q0 += 32) {
+            const int32_t q = q0 + lane;
+            if (q < w1 && q != x) {
+                const ARec<I, W> oq = cp.AR[q];
+                if (is_short(oq) && overlaps(oq, me) && precedes(me, oq) && (last || precedes(oq, R1)) &&
+                    atomicSub(CNT + q, 1) == 1)
+                    push(q);
+            }
+        }
+        __syncwarp();
+    }
+    return mx;
+}
+
+// Gap search over P predecessors already sorted by offset (off(x), end(x)):
+// the gap before the x-th is its offset minus the largest end before it.
+// FIRST takes the lowest offset whose gap fits, BEST the smallest fitting gap
+// (the lowest offset on ties); with no fitting gap, the largest end.
+template <typename Off, typename End>
+__device__ int64_t sorted_gap(int32_t P, int64_t s, int32_t policy, Off&& off, End&& end, int64_t* red) {
+    const int32_t chunk = (P + blockDim.x - 1) / blockDim.x;
+    const int32_t k0 = min(P, (int32_t)threadIdx.x * chunk), k1 = min(P, k0 + chunk);
+    int64_t local = 0;
+    for (int32_t x = k0; x < k1; ++x) local = max(local, end(x));
+    int64_t top;
+    int64_t prev = block_excl_max(local, red, &top);
+    int64_t key = INT64_MAX, val = INT64_MAX;
+    for (int32_t x = k0; x < k1; ++x) {
+        const int64_t gl = off(x) - prev;
+        if (gl >= s) {
+            const int64_t kx = policy == MP_FIT_FIRST ? prev : gl;  // prev grows with x
+            if (kx < key || (kx == key && prev < val)) {
+                key = kx;
+                val = prev;
+            }
+        }
+        prev = max(prev, end(x));
+    }
+    block_min_pair(key, val, red);
+    return key == INT64_MAX ? top : val;
+}
+
+// Places the k-th long-lived member of a component (every lower rank placed)
+// with the whole CTA.  Its predecessors -- the short-lived members of its
+// window that precede it and every long-lived member of lower rank, hr[0, k),
+// that overlaps it -- are gathered, sorted by offset, and searched in one
+// pass.  With the data in shared memory the gather keeps their positions in
+// idx (2n entries); otherwise (offset, end) pairs, in the shared scratch
+// (sbuf, up to scap pairs) or else in bo / be.  Returns the offset (every
+// thread).
+template <typename I, typename W, bool kSmem>
+__device__ W place_heavy(const Comp<I, W>& cp, int32_t k, int32_t policy, int32_t* idx, W* sbuf, int32_t scap,
+                         int64_t* bo, int64_t* be, int64_t* red, int32_t* cnt) {
+    const unsigned full = 0xffffffffu;
+    const int lane = threadIdx.x & 31;
+    int32_t p;
+    const ARec<I, W> me = cp.long_rec(k, p);
+    const int32_t a = me.a, f = me.f;
+    const int64_t s = (int64_t)me.s;
+    int32_t w0, w1;
+    cp.window(me, w0, w1);
+    const int32_t nw = max(0, w1 - w0), ncand = nw + k;
+    if (threadIdx.x == 0) *cnt = 0;
+    __syncthreads();
+    for (int32_t x0 = (int32_t)(threadIdx.x & ~31u); x0 < ncand; x0 += blockDim.x) {  // warp-uniform rounds
+        const int32_t x = x0 + lane;
+        bool hit = false;
+        int32_t q = -1;
+        int64_t po = 0, pe = 0;
+        if (x < nw) {
+            q = w0 + x;
+            if (q != p) {
+                const ARec<I, W> o = cp.AR[q];
+                hit = (int32_t)o.f - (int32_t)o.a <= kLongLife && (int32_t)o.a < f && a < (int32_t)o.f &&
+                      precedes(o, me);
+                if (hit && !kSmem) {
+                    po = (int64_t)cp.OFFP[q];
+                    pe = po + (int64_t)o.s;
+                }
+            }
+        } else if (x < ncand) {
+            const ARec<I, W> o = cp.long_rec(x - nw, q);
+            hit = (int32_t)o.a < f && a < (int32_t)o.f;
+            if (hit && !kSmem) {
+                po = (int64_t)cp.long_off(x - nw, q);
+                pe = po + (int64_t)o.s;
+            }
+        }
+        const unsigned bal = __ballot_sync(full, hit);
+        if (bal) {
+            int32_t at = 0;
+            if (lane == 0) at = atomicAdd(cnt, __popc(bal));
+            at = __shfl_sync(full, at, 0) + __popc(bal & ((1u << lane) - 1u));
+            if (hit) {
+                if (kSmem) {
+                    idx[at] = q;
+                } else if (at < scap) {
+                    sbuf[2 * at] = (W)po;
+                    sbuf[2 * at + 1] = (W)pe;
+                } else {
+                    bo[at] = po;
+                    be[at] = pe;
+                }
+            }
+        }
+    }
+    __syncthreads();
+    const int32_t P = *cnt;
+    const int32_t plen = (int32_t)pow2_at_least(P);
+    int64_t off;
+    if (kSmem) {  // sort positions by offset (-1 pads sort last)
+        for (int32_t x = P + threadIdx.x; x < plen; x += blockDim.x) idx[x] = -1;
+        __syncthreads();
+        const W* O = cp.OFFP;
+        block_bitonic_sort(idx, plen, [&](int32_t x, int32_t y) { return y < 0 ? x >= 0 : (x >= 0 && O[x] < O[y]); });
+        off = sorted_gap(P, s, policy, [&](int32_t x) { return (int64_t)O[idx[x]]; },
+                         [&](int32_t x) { return (int64_t)O[idx[x]] + (int64_t)cp.AR[idx[x]].s; }, red);
+    } else if (plen <= scap) {  // sort the pairs in shared memory
+        for (int32_t x = P + threadIdx.x; x < plen; x += blockDim.x) {
+            sbuf[2 * x] = w_none<W>();
+            sbuf[2 * x + 1] = w_none<W>();
+        }
+        __syncthreads();
+        for (int32_t kk = 2; kk <= plen; kk <<= 1) {
+            for (int32_t j = kk >> 1; j > 0; j >>= 1) {
+                for (int32_t t = threadIdx.x; t < (plen >> 1); t += blockDim.x) {
+                    const int32_t lo = 2 * t - (t & (j - 1)), hi = lo + j;
+                    const bool up = (lo & kk) == 0;
+                    const W xo = sbuf[2 * lo], yo = sbuf[2 * hi];
+                    if (up ? yo < xo : xo < yo) {
+                        const W xe = sbuf[2 * lo + 1];
+                        sbuf[2 * lo] = yo;
+                        sbuf[2 * hi] = xo;
+                        sbuf[2 * lo + 1] = sbuf[2 * hi + 1];
+                        sbuf[2 * hi + 1] = xe;
+                    }
+                }
+                __syncthreads();
+            }
+        }
+        off = sorted_gap(P, s, policy, [&](int32_t x) { return (int64_t)sbuf[2 * x]; },
+                         [&](int32_t x) { return (int64_t)sbuf[2 * x + 1]; }, red);
+    } else {  // too many for the scratch: all pairs to bo / be, sorted there
+        for (int32_t x = threadIdx.x; x < min(P, scap); x += blockDim.x) {
+            bo[x] = (int64_t)sbuf[2 * x];
+            be[x] = (int64_t)sbuf[2 * x + 1];
+        }
+        for (int32_t x = P + threadIdx.x; x < plen; x += blockDim.x) {
+            bo[x] = INT64_MAX;
+            be[x] = INT64_MAX;
+        }
+        __syncthreads();
+        for (int32_t kk = 2; kk <= plen; kk <<= 1) {
+            for (int32_t j = kk >> 1; j > 0; j >>= 1) {
+                for (int32_t t = threadIdx.x; t < (plen >> 1); t += blockDim.x) {
+                    const int32_t lo = 2 * t - (t & (j - 1)), hi = lo + j;
+                    const bool up = (lo & kk) == 0;
+                    const int64_t xo = bo[lo], yo = bo[hi];
+                    if (up ? yo < xo : xo < yo) {
+                        const int64_t xe = be[lo];
+                        bo[lo] = yo;
+                        bo[hi] = xo;
+                        be[lo] = be[hi];
+                        be[hi] = xe;
+                    }
+                }
+                __syncthreads();
+            }
+        }
+        off = sorted_gap(P, s, policy, [&](int32_t x) { return bo[x]; }, [&](int32_t x) { return be[x]; }, red);
+    }
+    if (threadIdx.x == 0) {
+        cp.OFFP[p] = (W)off;
+        if (cp.staged) cp.st.off[k] = (W)off;
+    }
+    __syncthreads();
+    return (W)off;
 }
 
 // ------------------------------------------------------------- components
 
-// Size of the component starting at position p: distance to the next start
-// flag in SB (n positions, one bit each), or to n.
-__device__ __forceinline__ int32_t comp_size(const uint32_t* SB, int32_t p, int32_t n) {
+// Component lookups over the start flags SB (n positions, one bit each).
+// Traces of more than kWordWalk words have per-word tables instead of walks
+// over SB: LW[w] is the last start in words 0..w, and -NW[w] the first start
+// in words w.. (n if none); without tables both are null.
+constexpr int32_t kWordWalk = 32;
+
+// Start of the component holding position p.
+__device__ __forceinline__ int32_t comp_start(const uint32_t* SB, const int32_t* LW, int32_t p) {
+    int32_t w = p >> 5;
+    uint32_t m = SB[w] & (0xffffffffu >> (31 - (p & 31)));  // starts at or before p in its word
+    if (m) return (w << 5) + 31 - __clz(m);
+    if (LW) return LW[w - 1];  // position 0 starts a component, so w >= 1 here
+    while (m == 0) m = SB[--w];
+    return (w << 5) + 31 - __clz(m);
+}
+
+// Size of the component starting at position p: distance to the next start.
+__device__ __forceinline__ int32_t comp_size(const uint32_t* SB, const int32_t* NW, int32_t p, int32_t n) {
     int32_t w = p >> 5;
     const int32_t nwords = (n + 31) >> 5;
     uint32_t m = SB[w] & ~((2u << (p & 31)) - 1u);  // start flags after p in its word
+    if (m) return (w << 5) + __ffs(m) - 1 - p;
+    if (NW) return (w + 1 < nwords ? -NW[w + 1] : n) - p;
     while (m == 0) {
         if (++w >= nwords) return n - p;
         m = SB[w];
     }
     return (w << 5) + __ffs(m) - 1 - p;
+}
+
+// In-place inclusive prefix maximum of x[0, len) by the whole block; with
+// `reverse`, taken from x[len - 1] down to x[0].  red: >= 33 slots.
+__device__ void block_scan_max_i32(int32_t* x, int32_t len, bool reverse, int32_t* red) {
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+    int32_t carry = INT32_MIN;
+    for (int32_t base = 0; base < len; base += blockDim.x) {
+        const int32_t i = base + (int32_t)threadIdx.x;
+        const int32_t at = reverse ? len - 1 - i : i;
+        int32_t v = i < len ? x[at] : INT32_MIN;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int32_t u = __shfl_up_sync(0xffffffffu, v, o);
+            if (lane >= o) v = max(v, u);
+        }
+        if (lane == 31) red[w] = v;
+        __syncthreads();
+        if (w == 0) {
+            int32_t xi = lane < nw ? red[lane] : INT32_MIN;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int32_t u = __shfl_up_sync(0xffffffffu, xi, o);
+                if (lane >= o) xi = max(xi, u);
+            }
+            if (lane < nw) red[lane] = xi;
+        }
+        __syncthreads();
+        v = max(v, max(carry, w == 0 ? INT32_MIN : red[w - 1]));
+        if (i < len) x[at] = v;
+        carry = max(carry, red[nw - 1]);
+        __syncthreads();
+    }
 }
 
 // Size class of a component of c >= 2 tensors.
@@ -552,8 +963,8 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
     constexpr bool kWide = sizeof(W) == 8;
     extern __shared__ __align__(16) unsigned char smem_raw[];
     __shared__ int64_t red[72];
-    __shared__ int32_t s_cnt, s_bin[kBins], s_base[kBins + 1], s_bad;
-    __shared__ unsigned long long s_top, s_hi, s_lo, s_max, s_key, s_lbmax;
+    __shared__ int32_t s_cnt, s_tail, s_bin[kBins], s_base[kBins + 1], s_bad, s_fail;
+    __shared__ unsigned long long s_hi, s_lo, s_max, s_key, s_lbmax;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
     const int32_t policy = out.policy;
     int32_t* __restrict__ status = out.status;
@@ -571,13 +982,19 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
     W* D = reinterpret_cast<W*>(base + L.dprof);  // fused: before the records exist
     int32_t* BEND = reinterpret_cast<int32_t*>(base + L.bend);
     uint32_t* SB = reinterpret_cast<uint32_t*>(base + L.sb);
+    int32_t* WT = reinterpret_cast<int32_t*>(base + L.wt);
     int32_t* LST = reinterpret_cast<int32_t*>(base + L.lst);
     uint16_t* RP = reinterpret_cast<uint16_t*>(base + L.rp);
-    // CTA tier workspace: predecessor offsets / ends, then the priority-ordered records
+    // CTA tier workspace: a long-lived member's predecessors (offsets, ends),
+    // then (data in the workspace) a large component's priority order and
+    // long-lived ranks
     const size_t cap2 = (size_t)pow2_at_least(bt.max_tensors > 0 ? bt.max_tensors : 1);
     int64_t* bo = reinterpret_cast<int64_t*>(ws + buf_offset + (size_t)b * buf_stride);
     int64_t* be = bo + cap2;
-    SRec<I>* SR = reinterpret_cast<SRec<I>*>(be + cap2);
+    int32_t* ORD = kSmem ? reinterpret_cast<int32_t*>(base + L.ord) : reinterpret_cast<int32_t*>(be + cap2);
+    int32_t* HR = kSmem ? reinterpret_cast<int32_t*>(base + L.rp) : ORD + cap2;
+    int32_t* CNT = kSmem ? reinterpret_cast<int32_t*>(base + L.cnt) : HR + cap2;
+    int32_t* QUE = kSmem ? reinterpret_cast<int32_t*>(base + L.que) : CNT + cap2;
 
     // ---- clear the histogram (and the difference array)
     for (int t = threadIdx.x; t < T; t += blockDim.x) BEND[t] = 0;
@@ -586,6 +1003,7 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
     if (threadIdx.x < kBins) s_bin[threadIdx.x] = 0;
     if (threadIdx.x == 0) {
         s_bad = 0;
+        s_fail = 0;
         s_hi = s_lo = s_max = s_lbmax = 0;
         s_key = ~0ull;
     }
@@ -770,6 +1188,23 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
         }
     }
     __syncthreads();
+    const int32_t nwords = (n + 31) >> 5;
+    const int32_t* LW = nullptr;
+    const int32_t* NW = nullptr;
+    if (nwords > kWordWalk) {  // per-word tables of the last and the next component start
+        int32_t* lw = WT;
+        int32_t* nw = WT + nwords;
+        for (int32_t w = threadIdx.x; w < nwords; w += blockDim.x) {
+            const uint32_t m = SB[w];
+            lw[w] = m ? (w << 5) + 31 - __clz(m) : -1;
+            nw[w] = m ? -((w << 5) + __ffs(m) - 1) : -n;
+        }
+        __syncthreads();
+        block_scan_max_i32(lw, nwords, false, reinterpret_cast<int32_t*>(red));
+        block_scan_max_i32(nw, nwords, true, reinterpret_cast<int32_t*>(red));
+        LW = lw;
+        NW = nw;
+    }
 
     // ---- members, one thread per tensor: a single tensor is placed at 0; a
     // member of a component of 2..kThreadComp tensors gets its rank and
@@ -780,11 +1215,8 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
         const int32_t p = q0 + threadIdx.x;
         int bin = -1;
         if (p < n) {
-            int32_t w = p >> 5;
-            uint32_t m = SB[w] & (0xffffffffu >> (31 - (p & 31)));  // starts at or before p in its word
-            while (m == 0) m = SB[--w];                             // position 0 starts a component
-            const int32_t p0 = (w << 5) + 31 - __clz(m);
-            const int32_t c = comp_size(SB, p0, n);
+            const int32_t p0 = comp_start(SB, LW, p);
+            const int32_t c = comp_size(SB, NW, p0, n);
             if (c == 1) {
                 OFFP[p] = 0;
                 mx = max(mx, AR[p].s);
@@ -823,7 +1255,7 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
         const int32_t p = q0 + threadIdx.x;
         int bin = -1;
         if (p < n && ((SB[p >> 5] >> (p & 31)) & 1u)) {
-            const int32_t c = comp_size(SB, p, n);
+            const int32_t c = comp_size(SB, NW, p, n);
             if (c > 1) bin = comp_bin(c);
         }
         const unsigned grp = __match_any_sync(0xffffffffu, bin);
@@ -840,48 +1272,91 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
         const int32_t wb = s_base[kBinWarp], nwc = s_base[kBinCta] - wb;
         for (int32_t k = warp; k < nwc; k += nwarps) {
             const int32_t p0 = LST[wb + k];
-            const W e = place_warp(AR, OFFP, p0, comp_size(SB, p0, n), policy);
+            const W e = place_warp(AR, OFFP, p0, comp_size(SB, NW, p0, n), policy);
             mx = max(mx, e);
         }
         // the largest thread-tier components go to the last warp, which has
         // the fewest warp-tier components
         for (int32_t g = ((nwarps - 1 - warp) << 5) + lane; g < wb; g += blockDim.x) {
-            const int32_t p0 = LST[g], c = comp_size(SB, p0, n);
+            const int32_t p0 = LST[g], c = comp_size(SB, NW, p0, n);
             const W e = place_thread(AR, RP, OFFP, p0, c, policy);
             mx = max(mx, e);
         }
     }
 
-    // ---- large components, the whole CTA each (64-bit bytes)
+    // ---- large components, the whole CTA each: sorted into priority order;
+    // the long-lived members cut the order into runs of short-lived ones, which
+    // the warps place together, each long-lived one then by the whole CTA
     const int32_t xb = s_base[kBinCta], nx = s_base[kBins] - xb;
-    const CtaScratch sc{red, &s_cnt, &s_top};
-    for (int32_t q = 0; q < nx; ++q) {
-        const int32_t p0 = LST[xb + q], sz = comp_size(SB, p0, n);
+    W* scratch = nullptr;
+    const LongStage<W> st = long_stage<W>(smem_raw, &scratch);
+    for (int32_t qc = 0; qc < nx; ++qc) {
+        const int32_t p0 = LST[xb + qc], sz = comp_size(SB, NW, p0, n);
         const int32_t len = (int32_t)pow2_at_least(sz);
-        int32_t* idx = reinterpret_cast<int32_t*>(bo);  // the index list lives in bo while sorting
-        for (int32_t x = threadIdx.x; x < len; x += blockDim.x) idx[x] = x < sz ? p0 + x : -1;
+        // len entries: with the data in shared memory, the rp and ord regions
+        // together (2n entries); the ranks and the order below only overwrite
+        // entries already read
+        int32_t* sortbuf = kSmem ? reinterpret_cast<int32_t*>(base + L.rp) : ORD;
+        __syncthreads();  // the thread tier's RP is dead
+        for (int32_t x = threadIdx.x; x < len; x += blockDim.x) sortbuf[x] = x < sz ? p0 + x : -1;
         __syncthreads();
-        block_bitonic_sort(idx, len, [&](int32_t x, int32_t y) {  // sentinels (-1) sort last
+        block_bitonic_sort(sortbuf, len, [&](int32_t x, int32_t y) {  // sentinels (-1) sort last
             return y < 0 ? x >= 0 : (x >= 0 && precedes(AR[x], AR[y]));
         });
-        for (int32_t x = threadIdx.x; x < sz; x += blockDim.x) {
-            const int32_t p = idx[x];
-            const ARec<I, W> me = AR[p];
-            SRec<I> rec;
-            rec.s = (int64_t)me.s;
-            rec.off = 0;
-            rec.a = me.a;
-            rec.f = me.f;
-            rec.id = me.id;
-            rec.pos = (I)p;
-            SR[x] = rec;
+        int32_t nl = 0;
+        for (int32_t r0 = 0; r0 < sz; r0 += blockDim.x) {
+            const int32_t r = r0 + threadIdx.x;
+            ARec<I, W> rx;
+            int32_t flag = 0;
+            if (r < sz) {
+                const int32_t px = sortbuf[r];
+                if constexpr (kSmem) ORD[r] = px;
+                rx = AR[px];
+                flag = (int32_t)rx.f - (int32_t)rx.a > kLongLife ? 1 : 0;
+            }
+            int32_t tot;
+            const int32_t at = nl + block_excl_scan<int32_t>(flag, reinterpret_cast<int32_t*>(red), &tot);
+            if (flag) {
+                HR[at] = r;
+                if (!kSmem && at < kLongStage) {
+                    st.s[at] = rx.s;
+                    st.a[at] = rx.a;
+                    st.f[at] = rx.f;
+                    st.id[at] = rx.id;
+                }
+            }
+            nl += tot;
         }
         __syncthreads();
-        place_large(SR, sz, policy, bo, be, sc);
-        for (int32_t x = threadIdx.x; x < sz; x += blockDim.x) {
-            const W o = (W)SR[x].off;
-            OFFP[SR[x].pos] = o;
-            mx = max(mx, (W)(o + (W)SR[x].s));
+        Comp<I, W> cp;
+        cp.AR = AR;
+        cp.OFFP = OFFP;
+        cp.BEND = BEND;
+        cp.ord = ORD;
+        cp.hr = HR;
+        cp.p0 = p0;
+        cp.c = sz;
+        cp.nl = nl;
+        cp.st = st;
+        cp.staged = !kSmem && nl <= kLongStage;
+        for (int32_t k = 0; k <= nl; ++k) {
+            const int32_t r0 = k == 0 ? 0 : HR[k - 1] + 1, r1 = k < nl ? HR[k] : sz;
+            if (r1 > r0) {  // the short-lived run between two long-lived members
+                const W e = place_run<I, W>(cp, r0, r1, k, CNT, QUE,
+                                            kSmem ? nullptr : scratch + (size_t)warp * kPredBuf * 2, policy, &s_cnt,
+                                            &s_tail, &s_fail);
+                mx = max(mx, e);
+                __syncthreads();
+            }
+            if (k < nl) {
+                const W o = place_heavy<I, W, kSmem>(cp, k, policy, CNT, scratch,
+                                                     kSmem ? 0 : (int32_t)(kScratchBytes / (2 * sizeof(W))), bo, be,
+                                                     red, &s_cnt);
+                if (threadIdx.x == 0) {
+                    int32_t q;
+                    mx = max(mx, (W)(o + cp.long_rec(k, q).s));
+                }
+            }
         }
         __syncthreads();
     }
@@ -889,6 +1364,7 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
     {
         const unsigned long long m = (unsigned long long)warp_max_w(mx);
         if (lane == 0 && m > 0) atomicMax(&s_max, m);
+        if (threadIdx.x == 0) s_cnt = 0;
     }
     __syncthreads();
 
@@ -896,12 +1372,33 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
     // pair once, from its earlier member in alloc order, is checked for address
     // overlap -- an independent pass over the alloc-ordered records
     if (kFused) {
+        // a thread per tensor; windows longer than kValWide go to a list (LST,
+        // free by now) and a warp each
         for (int32_t p = threadIdx.x; p < n; p += blockDim.x) {
             const ARec<I, W> ri = AR[p];
             const int32_t stop = BEND[ri.f - 1];  // tensors with alloc < free_i
             if (stop <= p + 1) continue;
+            if (stop - p - 1 > kValWide) {
+                LST[atomicAdd(&s_cnt, 1)] = p;
+                continue;
+            }
             const W oi = OFFP[p], ei = oi + ri.s;
             for (int32_t q = p + 1; q < stop; ++q) {
+                const W oj = OFFP[q];
+                if (oi < oj + AR[q].s && oj < ei) {
+                    const uint32_t i = (uint32_t)ri.id, j = (uint32_t)AR[q].id;
+                    atomicMin(&s_key, ((unsigned long long)(i < j ? i : j) << 32) | (i < j ? j : i));
+                }
+            }
+        }
+        __syncthreads();
+        const int32_t nwide = s_cnt;
+        for (int32_t k = warp; k < nwide; k += nwarps) {
+            const int32_t p = LST[k];
+            const ARec<I, W> ri = AR[p];
+            const int32_t stop = BEND[ri.f - 1];
+            const W oi = OFFP[p], ei = oi + ri.s;
+            for (int32_t q = p + 1 + lane; q < stop; q += 32) {
                 const W oj = OFFP[q];
                 if (oi < oj + AR[q].s && oj < ei) {
                     const uint32_t i = (uint32_t)ri.id, j = (uint32_t)AR[q].id;
@@ -927,7 +1424,7 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
                 out.conflict[2 * b + 1] = good ? -1 : (int32_t)(key & 0xffffffffu);
             }
         }
-        status[b] = MP_OK;
+        status[b] = s_fail ? MP_ETIMEOUT : MP_OK;
     }
 }
 
@@ -969,9 +1466,9 @@ PlanGeometry plan_geometry(const mp_batch& bt, bool fused) {
 
 // Workspace: the per-trace slices of the launches that keep their data there
 // (the two launches run one after the other and share it), then the CTA
-// tier's buffers per trace (predecessor offsets / ends, the index list of a
-// large component, and its records in priority order), sized for up to
-// max_tensors.
+// tier's buffers per trace (a long-lived member's predecessors; a large
+// component's priority order, long-lived ranks, predecessor counts and
+// ready queue), sized for up to max_tensors.
 struct PlanWorkspace {
     size_t buf_offset, buf_stride, total;
 };
@@ -982,10 +1479,9 @@ PlanWorkspace plan_workspace(const mp_batch& bt) {
         const PlanGeometry a = plan_geometry<uint32_t>(bt, fused), b = plan_geometry<int64_t>(bt, fused);
         slices = std::max(slices, std::max(a.data_stride, b.data_stride));
     }
-    const bool narrow = bt.max_tensors < 32767 && bt.max_steps <= 32767;
     const size_t cap2 = (size_t)pow2_at_least(bt.max_tensors > 0 ? bt.max_tensors : 1);
     w.buf_offset = (size_t)bt.n_traces * slices;
-    w.buf_stride = align_up(cap2 * 16 + (size_t)bt.max_tensors * (narrow ? sizeof(SRec<int16_t>) : sizeof(SRec<int32_t>)));
+    w.buf_stride = align_up(cap2 * 32);
     w.total = bt.n_traces == 0 ? 0 : w.buf_offset + (size_t)bt.n_traces * w.buf_stride;
     return w;
 }
@@ -993,10 +1489,10 @@ PlanWorkspace plan_workspace(const mp_batch& bt) {
 template <typename I, typename W, bool kSmem, bool kFused>
 cudaError_t launch_variant(const mp_batch& bt, const PlanGeometry& g, const PlanWorkspace& pw, const PlanOut& out,
                            unsigned char* ws, cudaStream_t stream) {
-    const size_t smem = kSmem ? g.data : 0;
-    const void* fn = (const void*)k_plan<I, W, kSmem, kFused>;
     const int threads = kSmem ? kPlanThreadsSmem : kPlanThreadsGlobal;
-    if (kSmem) {
+    const size_t smem = kSmem ? g.data : flow_smem_bytes<W>();
+    const void* fn = (const void*)k_plan<I, W, kSmem, kFused>;
+    {
         cudaError_t e = set_smem_limit(fn, smem);
         if (e != cudaSuccess) return e;
     }

@@ -52,7 +52,7 @@ def test_static_scratch_matches_workspace_entry_point(cuda_lib):
 def test_static_scratch_rejects_oversized_batch(cuda_lib):
     import paper_2203_00448_gb300 as mp
 
-    ts = tg.config(2)  # needs about 33.5 MB of scratch, more than the 16 MiB array
+    ts = tg.random_batch(0, 8192, 512, 1024)  # needs 32 MiB of scratch, more than the 16 MiB array
     db = mp.DeviceBatch.from_host(ts, "cuda")
     assert mp.plan_workspace_bytes(db) > 16 << 20
     rc, off, pk, st = _static_plan(cuda_lib, db, mp.FIT_FIRST)
