@@ -19,6 +19,7 @@ constexpr int kReplayThreads = 256;
 constexpr int kBreadthThreads = 128;
 constexpr int kPlanThreadsSmem = 128;    // one CTA per trace, data in shared memory
 constexpr int kPlanThreadsGlobal = 1024; // one CTA per trace, data in the workspace
+constexpr int kPlanThreadsWide = 512;    // the 64-bit launch: deferred traces, CTA tier included
 
 // Largest dynamic shared memory a kernel of this library requests per CTA
 // (sm_103a allows 227 KB); above it a kernel keeps its data in the workspace.
@@ -29,6 +30,9 @@ constexpr size_t kPlanSmemLimit = kSmemCeiling;
 
 // Raises the kernel's dynamic shared memory ceiling once per device.
 cudaError_t set_smem_limit(const void* func, size_t bytes);
+// Asks for the largest shared-memory carveout for func (once per device), so
+// that kernels launched back to back keep one L1 / shared split.
+cudaError_t prefer_shared(const void* func);
 
 // CTAs of `func` (threads, dynamic shared memory smem) the current device holds
 // at once: SM count x resident CTAs per SM (at least 1); cached per device.

@@ -72,6 +72,8 @@ constexpr int32_t kPredBuf = 128;    // CTA tier, data in the workspace: predece
 constexpr int32_t kLongStage = 2048; // CTA tier, data in the workspace: long-lived members staged in shared memory
 constexpr long long kSpinCycles = 1ll << 31;  // a wait for another warp longer than this is a fault
 constexpr int32_t kValWide = 64;     // validation: windows longer than this get a warp each
+constexpr int32_t kDeferComp = 256;  // the 32-bit launch defers traces with a component larger than this
+constexpr int32_t kSpinPolls = 64;   // polls of a queue slot before the waiting warp starts to sleep between them
 constexpr int32_t kDeferred = -1;    // trace status between the two launches: needs 64-bit bytes
 
 // Component size classes for the counting sort of the component list:
@@ -131,6 +133,7 @@ template <typename I, typename W>
 struct PlanLayout {
     size_t arec, offp, dprof, bend, sb, wt, lst, rp, ord, cnt, que, total;
     __host__ __device__ PlanLayout(int64_t n, int64_t T, bool fused) {
+        constexpr bool cta_tier = true;
         arec = 0;
         offp = arec + align16((size_t)n * sizeof(ARec<I, W>));
         const size_t main_end = offp + align16((size_t)n * sizeof(W));
@@ -140,11 +143,11 @@ struct PlanLayout {
         sb = bend + align16((size_t)T * 4);
         wt = sb + align16((size_t)((n + 31) / 32) * 4);
         lst = wt + align16((size_t)((n + 31) / 32) * 8);
-        rp = lst + align16((size_t)n * 4);   // later the CTA tier's long-lived ranks (int32)
-        ord = rp + align16((size_t)n * 4);   // the CTA tier's priority order (int32)
-        cnt = ord + align16((size_t)n * 4);  // the CTA tier's predecessor counts (int32)
-        que = cnt + align16((size_t)n * 4);  // the CTA tier's ready queue (int32)
-        total = align_up(que + align16((size_t)n * 4));
+        rp = lst + align16((size_t)n * 4);  // the thread tier's ranks; later the CTA tier's long-lived ranks
+        ord = rp + align16((size_t)n * (cta_tier ? 4 : 2));  // the CTA tier's priority order (int32)
+        cnt = ord + (cta_tier ? align16((size_t)n * 4) : 0);  // the CTA tier's predecessor counts (int32)
+        que = cnt + (cta_tier ? align16((size_t)n * 4) : 0);  // the CTA tier's ready queue (int32)
+        total = align_up(que + (cta_tier ? align16((size_t)n * 4) : 0));
     }
 };
 
@@ -408,8 +411,8 @@ __device__ __forceinline__ int32_t wait_slot(const volatile int32_t* slot, volat
     int32_t v = *slot;
     if (v >= 0) return v;
     const long long t0 = clock64();
-    for (;;) {
-        __nanosleep(64);
+    for (int32_t polls = 0;; ++polls) {
+        if (polls >= kSpinPolls) __nanosleep(32);  // a short wait is the common case: poll first
         v = *slot;
         if (v >= 0) return v;
         if (*fail || clock64() - t0 > kSpinCycles) {
@@ -536,7 +539,6 @@ __device__ W place_run(const Comp<I, W>& cp, int32_t r0, int32_t r1, int32_t nl_
         const int32_t at = atomicAdd(tail, 1);
         vque[at] = x;
     };
-
     // predecessors inside the run, a warp per member
     for (int32_t r = r0 + warp; r < r1; r += nwarps) {
         const int32_t x = cp.ord[r];
@@ -802,7 +804,22 @@ __device__ W place_heavy(const Comp<I, W>& cp, int32_t k, int32_t policy, int32_
     const int32_t P = *cnt;
     const int32_t plen = (int32_t)pow2_at_least(P);
     int64_t off;
-    if (kSmem) {  // sort positions by offset (-1 pads sort last)
+    if (kSmem && policy == MP_FIT_FIRST) {  // jump over the gathered positions
+        const W* O = cp.OFFP;
+        int64_t o = 0;
+        for (;;) {
+            int64_t next = o;
+            for (int32_t x = threadIdx.x; x < P; x += blockDim.x) {
+                const int32_t q = idx[x];
+                const int64_t po = (int64_t)O[q], pe = po + (int64_t)cp.AR[q].s;
+                if (po < o + s && o < pe && pe > next) next = pe;
+            }
+            next = block_max_i64(next, red);
+            if (next == o) break;
+            o = next;
+        }
+        off = o;
+    } else if (kSmem) {  // sort positions by offset (-1 pads sort last)
         for (int32_t x = P + threadIdx.x; x < plen; x += blockDim.x) idx[x] = -1;
         __syncthreads();
         const W* O = cp.OFFP;
@@ -953,6 +970,96 @@ __device__ __forceinline__ W block_excl_scan_w(W v, int64_t* red, W* total) {
     return block_excl_scan<W>(v, reinterpret_cast<W*>(red), total);
 }
 
+// Places the nx large components starting at LST[0, nx) with the whole CTA
+// (the 32-bit launch defers traces with components above kDeferComp).  Each
+// is sorted into priority order; its long-lived members cut the order into
+// runs of short-lived ones, which the warps place together, each long-lived
+// one then by the whole CTA.  sort_smem: 2n entries of shared memory for
+// the sort when the data is there.  Returns this thread's largest end.
+template <typename I, typename W, bool kSmem>
+__device__ __forceinline__ W large_tier(const ARec<I, W>* AR, W* OFFP, const int32_t* BEND, const uint32_t* SB,
+                                     const int32_t* NW, const int32_t* LST, int32_t nx, int32_t n, int32_t* sort_smem,
+                                     int32_t* ORD, int32_t* HR, int32_t* CNT, int32_t* QUE, int64_t* bo, int64_t* be,
+                                     unsigned char* smem_raw, int32_t policy, int64_t* red, int32_t* s_cnt,
+                                     int32_t* s_tail, int32_t* s_fail) {
+    const int warp = threadIdx.x >> 5;
+    W mx = 0;
+    W* scratch = nullptr;
+    const LongStage<W> st = long_stage<W>(smem_raw, &scratch);
+    for (int32_t qc = 0; qc < nx; ++qc) {
+        const int32_t p0 = LST[qc], sz = comp_size(SB, NW, p0, n);
+        const int32_t len = (int32_t)pow2_at_least(sz);
+        // len entries: with the data in shared memory, the rp and ord regions
+        // together (2n entries); the ranks and the order below only overwrite
+        // entries already read
+        int32_t* sortbuf = kSmem ? sort_smem : ORD;
+        __syncthreads();  // the thread tier's RP is dead
+        for (int32_t x = threadIdx.x; x < len; x += blockDim.x) sortbuf[x] = x < sz ? p0 + x : -1;
+        __syncthreads();
+        block_bitonic_sort(sortbuf, len, [&](int32_t x, int32_t y) {  // sentinels (-1) sort last
+            return y < 0 ? x >= 0 : (x >= 0 && precedes(AR[x], AR[y]));
+        });
+        int32_t nl = 0;
+        for (int32_t r0 = 0; r0 < sz; r0 += blockDim.x) {
+            const int32_t r = r0 + threadIdx.x;
+            ARec<I, W> rx;
+            int32_t flag = 0;
+            if (r < sz) {
+                const int32_t px = sortbuf[r];
+                if constexpr (kSmem) ORD[r] = px;
+                rx = AR[px];
+                flag = (int32_t)rx.f - (int32_t)rx.a > kLongLife ? 1 : 0;
+            }
+            int32_t tot;
+            const int32_t at = nl + block_excl_scan<int32_t>(flag, reinterpret_cast<int32_t*>(red), &tot);
+            if (flag) {
+                HR[at] = r;
+                if (!kSmem && at < kLongStage) {
+                    st.s[at] = rx.s;
+                    st.a[at] = rx.a;
+                    st.f[at] = rx.f;
+                    st.id[at] = rx.id;
+                }
+            }
+            nl += tot;
+        }
+        __syncthreads();
+        Comp<I, W> cp;
+        cp.AR = AR;
+        cp.OFFP = OFFP;
+        cp.BEND = BEND;
+        cp.ord = ORD;
+        cp.hr = HR;
+        cp.p0 = p0;
+        cp.c = sz;
+        cp.nl = nl;
+        cp.st = st;
+        cp.staged = !kSmem && nl <= kLongStage;
+        for (int32_t k = 0; k <= nl; ++k) {
+            const int32_t r0 = k == 0 ? 0 : HR[k - 1] + 1, r1 = k < nl ? HR[k] : sz;
+            if (r1 > r0) {  // the short-lived run between two long-lived members
+                const W e = place_run<I, W>(cp, r0, r1, k, CNT, QUE,
+                                            kSmem ? nullptr : scratch + (size_t)warp * kPredBuf * 2, policy, s_cnt,
+                                            s_tail, s_fail);
+                mx = max(mx, e);
+                __syncthreads();
+            }
+            if (k < nl) {
+                const W o = place_heavy<I, W, kSmem>(cp, k, policy, CNT, scratch,
+                                                     kSmem ? 0 : (int32_t)(kScratchBytes / (2 * sizeof(W))), bo, be,
+                                                     red, s_cnt);
+                if (threadIdx.x == 0) {
+                    int32_t q;
+                    mx = max(mx, (W)(o + cp.long_rec(k, q).s));
+                }
+            }
+        }
+        __syncthreads();
+    }
+
+    return mx;
+}
+
 // ------------------------------------------------------------- the kernel
 
 // The whole path for trace b, by the whole CTA.
@@ -963,7 +1070,7 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
     constexpr bool kWide = sizeof(W) == 8;
     extern __shared__ __align__(16) unsigned char smem_raw[];
     __shared__ int64_t red[72];
-    __shared__ int32_t s_cnt, s_tail, s_bin[kBins], s_base[kBins + 1], s_bad, s_fail;
+    __shared__ int32_t s_cnt, s_tail, s_bin[kBins], s_base[kBins + 1], s_bad, s_fail, s_big;
     __shared__ unsigned long long s_hi, s_lo, s_max, s_key, s_lbmax;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
     const int32_t policy = out.policy;
@@ -1004,6 +1111,7 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
     if (threadIdx.x == 0) {
         s_bad = 0;
         s_fail = 0;
+        s_big = 0;
         s_hi = s_lo = s_max = s_lbmax = 0;
         s_key = ~0ull;
     }
@@ -1221,7 +1329,10 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
                 OFFP[p] = 0;
                 mx = max(mx, AR[p].s);
             } else {
-                if (p == p0) bin = comp_bin(c);
+                if (p == p0) {
+                    bin = comp_bin(c);
+                    if (c > kDeferComp) s_big = 1;
+                }
                 if (c <= kThreadComp) {
                     const ARec<I, W> me = AR[p];
                     constexpr bool kPacked = sizeof(W) == 4 && sizeof(I) == 2;
@@ -1251,6 +1362,12 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
         if (lane == kBins - 1) s_base[kBins] = incl;
     }
     __syncthreads();
+    if constexpr (!kWide) {
+        if (s_big) {  // a component for the larger CTAs of the 64-bit launch
+            if (threadIdx.x == 0) status[b] = kDeferred;
+            return;
+        }
+    }
     for (int32_t q0 = 0; q0 < n; q0 += blockDim.x) {
         const int32_t p = q0 + threadIdx.x;
         int bin = -1;
@@ -1284,81 +1401,12 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
         }
     }
 
-    // ---- large components, the whole CTA each: sorted into priority order;
-    // the long-lived members cut the order into runs of short-lived ones, which
-    // the warps place together, each long-lived one then by the whole CTA
-    const int32_t xb = s_base[kBinCta], nx = s_base[kBins] - xb;
-    W* scratch = nullptr;
-    const LongStage<W> st = long_stage<W>(smem_raw, &scratch);
-    for (int32_t qc = 0; qc < nx; ++qc) {
-        const int32_t p0 = LST[xb + qc], sz = comp_size(SB, NW, p0, n);
-        const int32_t len = (int32_t)pow2_at_least(sz);
-        // len entries: with the data in shared memory, the rp and ord regions
-        // together (2n entries); the ranks and the order below only overwrite
-        // entries already read
-        int32_t* sortbuf = kSmem ? reinterpret_cast<int32_t*>(base + L.rp) : ORD;
-        __syncthreads();  // the thread tier's RP is dead
-        for (int32_t x = threadIdx.x; x < len; x += blockDim.x) sortbuf[x] = x < sz ? p0 + x : -1;
-        __syncthreads();
-        block_bitonic_sort(sortbuf, len, [&](int32_t x, int32_t y) {  // sentinels (-1) sort last
-            return y < 0 ? x >= 0 : (x >= 0 && precedes(AR[x], AR[y]));
-        });
-        int32_t nl = 0;
-        for (int32_t r0 = 0; r0 < sz; r0 += blockDim.x) {
-            const int32_t r = r0 + threadIdx.x;
-            ARec<I, W> rx;
-            int32_t flag = 0;
-            if (r < sz) {
-                const int32_t px = sortbuf[r];
-                if constexpr (kSmem) ORD[r] = px;
-                rx = AR[px];
-                flag = (int32_t)rx.f - (int32_t)rx.a > kLongLife ? 1 : 0;
-            }
-            int32_t tot;
-            const int32_t at = nl + block_excl_scan<int32_t>(flag, reinterpret_cast<int32_t*>(red), &tot);
-            if (flag) {
-                HR[at] = r;
-                if (!kSmem && at < kLongStage) {
-                    st.s[at] = rx.s;
-                    st.a[at] = rx.a;
-                    st.f[at] = rx.f;
-                    st.id[at] = rx.id;
-                }
-            }
-            nl += tot;
-        }
-        __syncthreads();
-        Comp<I, W> cp;
-        cp.AR = AR;
-        cp.OFFP = OFFP;
-        cp.BEND = BEND;
-        cp.ord = ORD;
-        cp.hr = HR;
-        cp.p0 = p0;
-        cp.c = sz;
-        cp.nl = nl;
-        cp.st = st;
-        cp.staged = !kSmem && nl <= kLongStage;
-        for (int32_t k = 0; k <= nl; ++k) {
-            const int32_t r0 = k == 0 ? 0 : HR[k - 1] + 1, r1 = k < nl ? HR[k] : sz;
-            if (r1 > r0) {  // the short-lived run between two long-lived members
-                const W e = place_run<I, W>(cp, r0, r1, k, CNT, QUE,
-                                            kSmem ? nullptr : scratch + (size_t)warp * kPredBuf * 2, policy, &s_cnt,
-                                            &s_tail, &s_fail);
-                mx = max(mx, e);
-                __syncthreads();
-            }
-            if (k < nl) {
-                const W o = place_heavy<I, W, kSmem>(cp, k, policy, CNT, scratch,
-                                                     kSmem ? 0 : (int32_t)(kScratchBytes / (2 * sizeof(W))), bo, be,
-                                                     red, &s_cnt);
-                if (threadIdx.x == 0) {
-                    int32_t q;
-                    mx = max(mx, (W)(o + cp.long_rec(k, q).s));
-                }
-            }
-        }
-        __syncthreads();
+    // ---- large components, the whole CTA each
+    if (s_base[kBins] > s_base[kBinCta]) {
+        const W e = large_tier<I, W, kSmem>(AR, OFFP, BEND, SB, NW, LST + s_base[kBinCta], s_base[kBins] - s_base[kBinCta],
+                                            n, kSmem ? reinterpret_cast<int32_t*>(base + L.rp) : nullptr, ORD, HR, CNT,
+                                            QUE, bo, be, smem_raw, policy, red, &s_cnt, &s_tail, &s_fail);
+        mx = max(mx, e);
     }
 
     {
@@ -1430,18 +1478,34 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
 
 // 32-bit launch: one CTA per trace.  64-bit launch: a grid no larger than
 // what the GPU holds at once walks every trace and takes the ones the 32-bit
-// launch deferred.
+// launch deferred (sizes summing to 2^32 or more, or a component of more
+// than kDeferComp tensors), with larger CTAs for the CTA tier.
 template <typename I, typename W, bool kSmem, bool kFused>
-__global__ void __launch_bounds__(kSmem ? kPlanThreadsSmem : kPlanThreadsGlobal, kSmem ? 9 : 1)
+__global__ void __launch_bounds__(sizeof(W) == 8 ? kPlanThreadsWide : (kSmem ? kPlanThreadsSmem : kPlanThreadsGlobal),
+                                  sizeof(W) == 8 ? 1 : (kSmem ? 9 : 1))
 k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_stride, size_t buf_offset,
        size_t buf_stride) {
     if constexpr (sizeof(W) == 4) {
         plan_trace<I, W, kSmem, kFused>(blockIdx.x, bt, out, ws, data_stride, buf_offset, buf_stride);
     } else {
-        for (int b = blockIdx.x; b < bt.n_traces; b += gridDim.x) {
-            if (out.status[b] != kDeferred) continue;
-            plan_trace<I, W, kSmem, kFused>(b, bt, out, ws, data_stride, buf_offset, buf_stride);
+        // this CTA's traces are blockIdx.x + k * gridDim.x; their statuses are
+        // read 32 at a time by one warp
+        __shared__ unsigned s_deferred;
+        for (int64_t k0 = 0; blockIdx.x + k0 * gridDim.x < bt.n_traces; k0 += 32) {
+            if (threadIdx.x < 32) {
+                const int64_t b = blockIdx.x + (k0 + threadIdx.x) * gridDim.x;
+                const unsigned m = __ballot_sync(0xffffffffu, b < bt.n_traces && out.status[b] == kDeferred);
+                if (threadIdx.x == 0) s_deferred = m;
+            }
             __syncthreads();
+            unsigned m = s_deferred;
+            __syncthreads();
+            while (m) {
+                const int b = (int)(blockIdx.x + (k0 + __ffs(m) - 1) * gridDim.x);
+                m &= m - 1;
+                plan_trace<I, W, kSmem, kFused>(b, bt, out, ws, data_stride, buf_offset, buf_stride);
+                __syncthreads();
+            }
         }
     }
 }
@@ -1489,11 +1553,12 @@ PlanWorkspace plan_workspace(const mp_batch& bt) {
 template <typename I, typename W, bool kSmem, bool kFused>
 cudaError_t launch_variant(const mp_batch& bt, const PlanGeometry& g, const PlanWorkspace& pw, const PlanOut& out,
                            unsigned char* ws, cudaStream_t stream) {
-    const int threads = kSmem ? kPlanThreadsSmem : kPlanThreadsGlobal;
-    const size_t smem = kSmem ? g.data : flow_smem_bytes<W>();
+    const int threads = sizeof(W) == 8 ? kPlanThreadsWide : (kSmem ? kPlanThreadsSmem : kPlanThreadsGlobal);
+    const size_t smem = kSmem ? g.data : (sizeof(W) == 8 ? flow_smem_bytes<W>() : 0);
     const void* fn = (const void*)k_plan<I, W, kSmem, kFused>;
     {
         cudaError_t e = set_smem_limit(fn, smem);
+        if (e == cudaSuccess) e = prefer_shared(fn);
         if (e != cudaSuccess) return e;
     }
     int grid = bt.n_traces;
