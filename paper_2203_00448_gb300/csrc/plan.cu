@@ -72,6 +72,7 @@ constexpr int32_t kPredBuf = 128;    // CTA tier, data in the workspace: predece
 constexpr int32_t kLongStage = 2048; // CTA tier, data in the workspace: long-lived members staged in shared memory
 constexpr long long kSpinCycles = 1ll << 31;  // a wait for another warp longer than this is a fault
 constexpr int32_t kValWide = 64;     // validation: windows longer than this get a warp each
+constexpr int32_t kFlowWarps = 16;   // warps that take members from a run's ready queue
 constexpr int32_t kDeferComp = 256;  // the 32-bit launch defers traces with a component larger than this
 constexpr int32_t kSpinPolls = 64;   // polls of a queue slot before the waiting warp starts to sleep between them
 constexpr int32_t kDeferred = -1;    // trace status between the two launches: needs 64-bit bytes
@@ -564,6 +565,7 @@ __device__ W place_run(const Comp<I, W>& cp, int32_t r0, int32_t r1, int32_t nl_
 
     W mx = 0;
     for (;;) {
+        if (warp >= kFlowWarps) break;  // the rest wait at the barrier instead of polling the queue
         int32_t idx = 0;
         if (lane == 0) idx = atomicAdd(head, 1);
         idx = __shfl_sync(full, idx, 0);
@@ -739,11 +741,12 @@ __device__ int64_t sorted_gap(int32_t P, int64_t s, int32_t policy, Off&& off, E
 // Places the k-th long-lived member of a component (every lower rank placed)
 // with the whole CTA.  Its predecessors -- the short-lived members of its
 // window that precede it and every long-lived member of lower rank, hr[0, k),
-// that overlaps it -- are gathered, sorted by offset, and searched in one
-// pass.  With the data in shared memory the gather keeps their positions in
-// idx (2n entries); otherwise (offset, end) pairs, in the shared scratch
-// (sbuf, up to scap pairs) or else in bo / be.  Returns the offset (every
-// thread).
+// that overlaps it -- are gathered: with the data in shared memory as
+// positions in idx (2n entries), otherwise as (offset, end) pairs in the
+// shared scratch (sbuf, up to scap pairs) or else in bo / be.  FIRST then
+// jumps to the largest conflicting end until nothing conflicts (a block
+// reduction per jump); BEST sorts them by offset and searches the gaps in
+// one pass.  Returns the offset (every thread).
 template <typename I, typename W, bool kSmem>
 __device__ W place_heavy(const Comp<I, W>& cp, int32_t k, int32_t policy, int32_t* idx, W* sbuf, int32_t scap,
                          int64_t* bo, int64_t* be, int64_t* red, int32_t* cnt) {
@@ -812,6 +815,20 @@ __device__ W place_heavy(const Comp<I, W>& cp, int32_t k, int32_t policy, int32_
             for (int32_t x = threadIdx.x; x < P; x += blockDim.x) {
                 const int32_t q = idx[x];
                 const int64_t po = (int64_t)O[q], pe = po + (int64_t)cp.AR[q].s;
+                if (po < o + s && o < pe && pe > next) next = pe;
+            }
+            next = block_max_i64(next, red);
+            if (next == o) break;
+            o = next;
+        }
+        off = o;
+    } else if (policy == MP_FIT_FIRST) {  // jump over the gathered pairs
+        int64_t o = 0;
+        for (;;) {
+            int64_t next = o;
+            for (int32_t x = threadIdx.x; x < P; x += blockDim.x) {
+                const int64_t po = x < scap ? (int64_t)sbuf[2 * x] : bo[x];
+                const int64_t pe = x < scap ? (int64_t)sbuf[2 * x + 1] : be[x];
                 if (po < o + s && o < pe && pe > next) next = pe;
             }
             next = block_max_i64(next, red);
