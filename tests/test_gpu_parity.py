@@ -123,6 +123,29 @@ def test_global_memory_path(cuda_lib, name, pol):
     assert_parity(ts, gpu_run(ts, name), oracle_run(ts, pol))
 
 
+@pytest.mark.parametrize("name,pol", POLICIES)
+def test_long_lived_chain_workspace_path(cuda_lib, name, pol):
+    """One component of 14,000 tensors that all live longer than 32 steps, on
+    the workspace variant: the long-lived list is too long to stage in shared
+    memory, and every member is placed by the whole CTA.  A second trace
+    mixes short-lived members with about 200 long-lived ones around them, so
+    that short-lived members gather more than 128 predecessors."""
+    rng = np.random.default_rng(11)
+    n = 14000
+    a = np.arange(n) // 2
+    T = int(a[-1]) + 80
+    f = np.minimum(a + rng.integers(33, 70, size=n), T)
+    s = rng.integers(1, 1 << 12, size=n) * 64
+    n2, T2 = 3000, 1200
+    a2 = rng.integers(0, T2, size=n2)
+    f2 = np.minimum(a2 + rng.integers(1, 4, size=n2), T2)
+    la = rng.integers(0, 100, size=200)
+    lf = np.minimum(la + rng.integers(900, 1200, size=200), T2)
+    s2 = rng.integers(1, 1 << 10, size=n2 + 200) * 4
+    ts = tg.from_arrays([(T, a, f, s), (T2, np.concatenate([a2, la]), np.concatenate([f2, lf]), s2)])
+    assert_parity(ts, gpu_run(ts, name), oracle_run(ts, pol))
+
+
 def test_empty_and_degenerate(cuda_lib):
     ts = tg.from_tuples([(0, []), (5, []), (1, [(0, 1, 1)]), (3, [(0, 3, 7), (0, 3, 7), (1, 2, 7)]),
                          (4, [(0, 4, 2 ** 40), (0, 4, 2 ** 40)])])
