@@ -68,12 +68,12 @@ constexpr int32_t kThreadComp = 8;   // components up to this size: one thread
 constexpr int32_t kWarpComp = 32;    // ... up to this size: one warp (a tensor per lane); else the CTA
 constexpr int kCached = 4;           // tensors per thread kept in registers between the two input passes
 constexpr int32_t kLongLife = 32;    // CTA tier: members living longer than this many steps are listed apart
-constexpr int32_t kPredBuf = 128;    // CTA tier, data in the workspace: predecessors gathered per warp
+constexpr int32_t kPredBuf = 512;    // CTA tier, data in the workspace: predecessors gathered per warp
 constexpr int32_t kLongStage = 2048; // CTA tier, data in the workspace: long-lived members staged in shared memory
 constexpr long long kSpinCycles = 1ll << 31;  // a wait for another warp longer than this is a fault
 constexpr int32_t kValWide = 64;     // validation: windows longer than this get a warp each
 constexpr int32_t kFlowWarps = 16;   // warps that take members from a run's ready queue
-constexpr int32_t kDeferComp = 256;  // the 32-bit launch defers traces with a component larger than this
+constexpr int32_t kDeferComp = 256;  // the 32-bit launch (data in shared memory) defers larger components
 constexpr int32_t kSpinPolls = 64;   // polls of a queue slot before the waiting warp starts to sleep between them
 constexpr int32_t kDeferred = -1;    // trace status between the two launches: needs 64-bit bytes
 
@@ -483,6 +483,8 @@ struct Comp {
 // warp while short-lived members are placed, the predecessors of a
 // long-lived member while it is placed.
 constexpr size_t kScratchBytes = 128 * 1024;
+static_assert((kPlanThreadsWide / 32) * kPredBuf * 2 * sizeof(int64_t) <= kScratchBytes,
+              "the per-warp predecessor buffers of the 64-bit launch fit in the scratch");
 template <typename W>
 __host__ __device__ constexpr size_t flow_smem_bytes() {
     return (size_t)kLongStage * (2 * sizeof(W) + 12) + kScratchBytes;
@@ -988,7 +990,8 @@ __device__ __forceinline__ W block_excl_scan_w(W v, int64_t* red, W* total) {
 }
 
 // Places the nx large components starting at LST[0, nx) with the whole CTA
-// (the 32-bit launch defers traces with components above kDeferComp).  Each
+// (the 32-bit launch defers traces with components above kDeferComp, and
+// with its data in the workspace, every trace that needs this tier).  Each
 // is sorted into priority order; its long-lived members cut the order into
 // runs of short-lived ones, which the warps place together, each long-lived
 // one then by the whole CTA.  sort_smem: 2n entries of shared memory for
@@ -1348,7 +1351,9 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
             } else {
                 if (p == p0) {
                     bin = comp_bin(c);
-                    if (c > kDeferComp) s_big = 1;
+                    // the 32-bit launch keeps the CTA tier only with its data in
+                    // shared memory and components up to kDeferComp
+                    if (c > (kSmem ? kDeferComp : kWarpComp)) s_big = 1;
                 }
                 if (c <= kThreadComp) {
                     const ARec<I, W> me = AR[p];
@@ -1495,8 +1500,8 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
 
 // 32-bit launch: one CTA per trace.  64-bit launch: a grid no larger than
 // what the GPU holds at once walks every trace and takes the ones the 32-bit
-// launch deferred (sizes summing to 2^32 or more, or a component of more
-// than kDeferComp tensors), with larger CTAs for the CTA tier.
+// launch deferred (sizes summing to 2^32 or more, or a component the 32-bit
+// launch does not place), with larger CTAs for the CTA tier.
 template <typename I, typename W, bool kSmem, bool kFused>
 __global__ void __launch_bounds__(sizeof(W) == 8 ? kPlanThreadsWide : (kSmem ? kPlanThreadsSmem : kPlanThreadsGlobal),
                                   sizeof(W) == 8 ? 1 : (kSmem ? 9 : 1))

@@ -146,6 +146,25 @@ def test_long_lived_chain_workspace_path(cuda_lib, name, pol):
     assert_parity(ts, gpu_run(ts, name), oracle_run(ts, pol))
 
 
+@pytest.mark.parametrize("name,pol", POLICIES)
+def test_mid_size_component_workspace_path(cuda_lib, name, pol):
+    """A batch too large for shared memory whose traces hold components of 33
+    to 256 tensors (placed by the CTA tier) among thousands of single ones."""
+    rng = np.random.default_rng(5)
+    traces = []
+    for c in (33, 100, 256):
+        n1, T = 13000, 16000
+        a1 = np.sort(rng.choice(T - 200, size=n1, replace=False))
+        a1 = a1[(a1 < 5000) | (a1 >= 5100)]  # keep clear of the block below
+        f1 = a1 + 1
+        a2 = 5000 + rng.integers(0, 10, size=c)
+        f2 = 5040 + rng.integers(0, 10, size=c)
+        s = rng.integers(1, 1 << 14, size=len(a1) + c) * 64
+        traces.append((T, np.concatenate([a1, a2]), np.concatenate([f1, f2]), s))
+    ts = tg.from_arrays(traces)
+    assert_parity(ts, gpu_run(ts, name), oracle_run(ts, pol))
+
+
 def test_empty_and_degenerate(cuda_lib):
     ts = tg.from_tuples([(0, []), (5, []), (1, [(0, 1, 1)]), (3, [(0, 3, 7), (0, 3, 7), (1, 2, 7)]),
                          (4, [(0, 4, 2 ** 40), (0, 4, 2 ** 40)])])
