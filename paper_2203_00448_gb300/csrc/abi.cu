@@ -29,19 +29,6 @@ cudaError_t set_smem_limit(const void* func, size_t bytes) {
     return e;
 }
 
-cudaError_t prefer_shared(const void* func) {
-    static std::mutex mu;
-    static std::set<std::pair<int, const void*>> done;
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return e;
-    std::lock_guard<std::mutex> lock(mu);
-    if (done.count({dev, func})) return cudaSuccess;
-    e = cudaFuncSetAttribute(func, cudaFuncAttributePreferredSharedMemoryCarveout, (int)cudaSharedmemCarveoutMaxShared);
-    if (e == cudaSuccess) done.insert({dev, func});
-    return e;
-}
-
 cudaError_t max_resident_ctas(const void* func, int threads, size_t smem, int* ctas) {
     static std::mutex mu;
     static std::map<std::tuple<int, const void*, int, size_t>, int> cache;

@@ -30,9 +30,6 @@ constexpr size_t kPlanSmemLimit = kSmemCeiling;
 
 // Raises the kernel's dynamic shared memory ceiling once per device.
 cudaError_t set_smem_limit(const void* func, size_t bytes);
-// Asks for the largest shared-memory carveout for func (once per device), so
-// that kernels launched back to back keep one L1 / shared split.
-cudaError_t prefer_shared(const void* func);
 
 // CTAs of `func` (threads, dynamic shared memory smem) the current device holds
 // at once: SM count x resident CTAs per SM (at least 1); cached per device.

@@ -1509,7 +1509,11 @@ k_plan(mp_batch bt, PlanOut out, unsigned char* __restrict__ ws, size_t data_str
        size_t buf_stride) {
     if constexpr (sizeof(W) == 4) {
         plan_trace<I, W, kSmem, kFused>(blockIdx.x, bt, out, ws, data_stride, buf_offset, buf_stride);
+        // the 64-bit launch may start now; it waits for this grid to finish
+        // (and its writes to land) before it reads anything this grid wrote
+        asm volatile("griddepcontrol.launch_dependents;");
     } else {
+        asm volatile("griddepcontrol.wait;" ::: "memory");
         // this CTA's traces are blockIdx.x + k * gridDim.x; their statuses are
         // read 32 at a time by one warp
         __shared__ unsigned s_deferred;
@@ -1580,7 +1584,6 @@ cudaError_t launch_variant(const mp_batch& bt, const PlanGeometry& g, const Plan
     const void* fn = (const void*)k_plan<I, W, kSmem, kFused>;
     {
         cudaError_t e = set_smem_limit(fn, smem);
-        if (e == cudaSuccess) e = prefer_shared(fn);
         if (e != cudaSuccess) return e;
     }
     int grid = bt.n_traces;
@@ -1590,9 +1593,25 @@ cudaError_t launch_variant(const mp_batch& bt, const PlanGeometry& g, const Plan
         if (e != cudaSuccess) return e;
         grid = std::max(1, std::min(grid, resident));
     }
-    k_plan<I, W, kSmem, kFused><<<(unsigned)grid, threads, smem, stream>>>(bt, out, ws, g.data_stride, pw.buf_offset,
-                                                                           pw.buf_stride);
-    return cudaGetLastError();
+    if (sizeof(W) == 4) {
+        k_plan<I, W, kSmem, kFused><<<(unsigned)grid, threads, smem, stream>>>(bt, out, ws, g.data_stride,
+                                                                               pw.buf_offset, pw.buf_stride);
+        return cudaGetLastError();
+    }
+    // the 64-bit launch depends on the 32-bit one programmatically: its CTAs
+    // may be scheduled while the first grid drains, and wait in-kernel
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3((unsigned)threads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, k_plan<I, W, kSmem, kFused>, bt, out, ws, g.data_stride, pw.buf_offset,
+                              pw.buf_stride);
 }
 
 template <typename W, bool kFused>
