@@ -10,7 +10,7 @@
 
 namespace mp {
 
-constexpr int kProfileThreads = 128;  // four traces per CTA, one warp each
+constexpr int kProfileThreads = 128;  // one CTA per trace
 constexpr int kValidateThreads = 128;
 constexpr int kPeakThreads = 256;
 constexpr int kBumpThreads = 128;

@@ -434,9 +434,11 @@ __device__ __forceinline__ int nth_set_bit(unsigned m, int n) {
 
 // A large component in the CTA tier.  Its members in priority order are
 // ord[0, c) (positions); the long-lived ones (life above kLongLife steps) are
-// at the ranks hr[0, nl), ascending.  A short-lived member x can only overlap
-// members allocated in (a_x - kLongLife, f_x) -- a window of alloc order
-// (BEND[t] = tensors allocated at or before t) -- or long-lived ones.  The
+// at the ranks hr[0, nl), ascending.  With lw the longest life among the
+// short-lived members (at most kLongLife), a short-lived member y overlaps x
+// only if a_y > a_x - lw, so x can only overlap short-lived members allocated
+// in (a_x - lw, f_x) -- a window of alloc order (BEND[t] = tensors allocated
+// at or before t) -- or long-lived ones.  The
 // variant with its data in the workspace stages the first kLongStage
 // long-lived members in shared memory, by list index.
 template <typename W>
@@ -454,12 +456,12 @@ struct Comp {
     const int32_t* BEND;
     const int32_t* ord;
     const int32_t* hr;
-    int32_t p0, c, nl;
+    int32_t p0, c, nl, lw;
     LongStage<W> st;
     bool staged;
 
     __device__ __forceinline__ void window(const ARec<I, W>& me, int32_t& w0, int32_t& w1) const {
-        w0 = max(p0, (int32_t)me.a >= kLongLife ? BEND[(int32_t)me.a - kLongLife] : 0);
+        w0 = max(p0, (int32_t)me.a >= lw ? BEND[(int32_t)me.a - lw] : 0);
         w1 = min(p0 + c, BEND[(int32_t)me.f - 1]);
     }
     // The k-th long-lived member (record and offset; the offset once placed).
@@ -1019,7 +1021,7 @@ __device__ __forceinline__ W large_tier(const ARec<I, W>* AR, W* OFFP, const int
         block_bitonic_sort(sortbuf, len, [&](int32_t x, int32_t y) {  // sentinels (-1) sort last
             return y < 0 ? x >= 0 : (x >= 0 && precedes(AR[x], AR[y]));
         });
-        int32_t nl = 0;
+        int32_t nl = 0, lw = 1;
         for (int32_t r0 = 0; r0 < sz; r0 += blockDim.x) {
             const int32_t r = r0 + threadIdx.x;
             ARec<I, W> rx;
@@ -1028,7 +1030,9 @@ __device__ __forceinline__ W large_tier(const ARec<I, W>* AR, W* OFFP, const int
                 const int32_t px = sortbuf[r];
                 if constexpr (kSmem) ORD[r] = px;
                 rx = AR[px];
-                flag = (int32_t)rx.f - (int32_t)rx.a > kLongLife ? 1 : 0;
+                const int32_t life = (int32_t)rx.f - (int32_t)rx.a;
+                flag = life > kLongLife ? 1 : 0;
+                if (!flag) lw = max(lw, life);
             }
             int32_t tot;
             const int32_t at = nl + block_excl_scan<int32_t>(flag, reinterpret_cast<int32_t*>(red), &tot);
@@ -1044,6 +1048,8 @@ __device__ __forceinline__ W large_tier(const ARec<I, W>* AR, W* OFFP, const int
             nl += tot;
         }
         __syncthreads();
+        int64_t lw_max;
+        block_excl_max((int64_t)lw, red, &lw_max);
         Comp<I, W> cp;
         cp.AR = AR;
         cp.OFFP = OFFP;
@@ -1053,6 +1059,7 @@ __device__ __forceinline__ W large_tier(const ARec<I, W>* AR, W* OFFP, const int
         cp.p0 = p0;
         cp.c = sz;
         cp.nl = nl;
+        cp.lw = (int32_t)lw_max;
         cp.st = st;
         cp.staged = !kSmem && nl <= kLongStage;
         for (int32_t k = 0; k <= nl; ++k) {

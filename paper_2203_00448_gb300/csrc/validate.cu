@@ -19,24 +19,124 @@ namespace mp {
 
 namespace {
 
-// Per-trace working set: tensors scattered into alloc-step order as packed
-// (offset, end) records with their id and free step, plus the bucket ends.
+// Per-trace working set: tensors scattered into alloc-step order as (offset,
+// end) records -- 8 bytes when every end of the trace is below 2^32, else 16
+// -- and (free step, id) pairs, plus the bucket ends.
 struct ValidateLayout {
-    size_t rec, id, fp, bend, total;
+    size_t rec, fi, bend, total;
     __host__ __device__ ValidateLayout(int64_t n, int64_t T) {
         rec = 0;
-        id = rec + align_up((size_t)n * 16);
-        fp = id + align_up((size_t)n * 4);
-        bend = fp + align_up((size_t)n * 4);
+        fi = rec + align_up((size_t)n * 16);
+        bend = fi + align_up((size_t)n * 8);
         total = bend + align_up((size_t)T * 4);
     }
 };
 
+// Per-trace flags, or-ed over the block.
+constexpr int kFlagInvalid = 1;  // a tensor breaks 0 <= a < f <= T, s >= 1, or has offset < 0
+constexpr int kFlagEndOvf = 2;   // offset + size past INT64_MAX
+constexpr int kFlagWide = 4;     // an end at or above 2^32
+constexpr int kFlagBigSize = 8;  // a size at or above 2^32: the size sum needs the exact check
+
 struct ValidateShared {
-    unsigned long long key, sum_hi, sum_lo;
-    int bad, ovf;
+    unsigned long long key;
+    unsigned int sum[3];  // the sizes' sum in three 21-bit limbs (carries kept)
+    int flags;
 };
 
+constexpr int kValCached = 4;  // tensors per thread held in registers between the two passes
+constexpr int kValItems = 8;   // bucket counts scanned per thread per tile
+
+// Adds a warp's per-lane saturated size sums into the three 21-bit limbs of
+// sum: every lane's limb is below 2^22, so a 32-bit warp reduction of each
+// cannot wrap, nor can the block's 32-bit shared sums (at most 32 warps).
+__device__ __forceinline__ void block_add_size_limbs(uint64_t v, unsigned int* sum) {
+    const unsigned full = 0xffffffffu;
+    const unsigned l0 = __reduce_add_sync(full, (unsigned)(v & 0x1fffffu));
+    const unsigned l1 = __reduce_add_sync(full, (unsigned)((v >> 21) & 0x1fffffu));
+    const unsigned l2 = __reduce_add_sync(full, (unsigned)(v >> 42));
+    if ((threadIdx.x & 31) == 0 && (l0 | l1 | l2)) {
+        atomicAdd(sum, l0);
+        atomicAdd(sum + 1, l1);
+        atomicAdd(sum + 2, l2);
+    }
+}
+
+// True if the limbs add up to more than INT64_MAX.
+__device__ __forceinline__ bool size_limbs_overflow(const unsigned int* sum) {
+    const uint64_t l0 = sum[0], l1 = sum[1] + (l0 >> 21), l2 = sum[2] + (l1 >> 21);
+    return l2 >= (1ull << 21);  // bits 42 and up reach 2^63
+}
+
+// In-place exclusive scan of the shared, 16-byte aligned x[0, len) by the
+// whole block, kValItems consecutive entries per thread per tile; ends with a
+// barrier.
+__device__ void block_excl_scan_i32(int32_t* x, int32_t len, int32_t* red) {
+    int32_t carry = 0;
+    const int32_t tile = (int32_t)blockDim.x * kValItems;
+    for (int32_t base = 0; base < len; base += tile) {
+        const int32_t my = base + (int32_t)threadIdx.x * kValItems;
+        const bool full = my + kValItems <= len;
+        int32_t v[kValItems];
+        if (full) {
+            const int4 u = *reinterpret_cast<const int4*>(x + my), w = *reinterpret_cast<const int4*>(x + my + 4);
+            v[0] = u.x, v[1] = u.y, v[2] = u.z, v[3] = u.w, v[4] = w.x, v[5] = w.y, v[6] = w.z, v[7] = w.w;
+        } else {
+#pragma unroll
+            for (int k = 0; k < kValItems; ++k) v[k] = my + k < len ? x[my + k] : 0;
+        }
+        int32_t sum = 0;
+#pragma unroll
+        for (int k = 0; k < kValItems; ++k) sum += v[k];
+        int32_t tot;
+        int32_t pre = block_excl_scan<int32_t>(sum, red, &tot) + carry;
+#pragma unroll
+        for (int k = 0; k < kValItems; ++k) {
+            const int32_t t = v[k];
+            v[k] = pre;
+            pre += t;
+        }
+        if (full) {
+            *reinterpret_cast<int4*>(x + my) = make_int4(v[0], v[1], v[2], v[3]);
+            *reinterpret_cast<int4*>(x + my + 4) = make_int4(v[4], v[5], v[6], v[7]);
+        } else {
+#pragma unroll
+            for (int k = 0; k < kValItems; ++k)
+                if (my + k < len) x[my + k] = v[k];
+        }
+        carry += tot;
+    }
+    __syncthreads();
+}
+
+// Every lifetime-overlapping pair once, from its earlier member in alloc
+// order (positions p < q < BEND[f_p - 1]); records R are (offset, end).
+template <typename R>
+__device__ __forceinline__ void check_pairs(const R* __restrict__ rec, const int2* __restrict__ fi_arr,
+                                            const int32_t* __restrict__ bend, int32_t n, unsigned long long* key) {
+    for (int32_t p = threadIdx.x; p < n; p += blockDim.x) {
+        const int2 fi = fi_arr[p];
+        const int32_t stop = bend[fi.x - 1];
+        if (stop <= p + 1) continue;
+        const R ri = rec[p];
+        for (int32_t q = p + 1; q < stop; ++q) {
+            const R rj = rec[q];
+            if (ri.x < rj.y && rj.x < ri.y) {
+                const uint32_t i = (uint32_t)fi.y, j = (uint32_t)fi_arr[q].y;
+                const uint32_t lo = i < j ? i : j, hi = i < j ? j : i;
+                atomicMin(key, ((unsigned long long)lo << 32) | hi);
+            }
+        }
+    }
+}
+
+// One CTA per trace.  The first kValCached * blockDim tensors are loaded into
+// registers before anything else (16-byte loads when the trace's slices are
+// aligned) and kept there for the scatter, so a trace's inputs are read from
+// memory once; larger traces read the rest twice.  Traces whose ends all lie
+// below 2^32 (the flag reduction tells) take 8-byte records and 32-bit
+// compares; the exact size sum is only formed when some size reaches 2^32
+// (below that, n < 2^31 sizes cannot sum past INT64_MAX).
 template <bool kSmem>
 __global__ void __launch_bounds__(kValidateThreads, kSmem ? 12 : 1)
 k_validate(mp_batch bt, const int64_t* __restrict__ offsets, int32_t* __restrict__ verdict,
@@ -52,64 +152,97 @@ k_validate(mp_batch bt, const int64_t* __restrict__ offsets, int32_t* __restrict
         return;
     }
     const int32_t n = tv.n, T = tv.T;
-    const ValidateLayout L(kSmem ? n : bt.max_tensors, kSmem ? T : bt.max_steps);
-    unsigned char* base = kSmem ? smem_raw : ws + (size_t)b * ws_stride;
-    longlong2* REC = reinterpret_cast<longlong2*>(base + L.rec);
-    int32_t* ID = reinterpret_cast<int32_t*>(base + L.id);
-    int32_t* FP = reinterpret_cast<int32_t*>(base + L.fp);
-    int32_t* BEND = reinterpret_cast<int32_t*>(base + L.bend);
-
-    for (int t = threadIdx.x; t < T; t += blockDim.x) BEND[t] = 0;
-    if (threadIdx.x == 0) {
-        sh.key = ~0ull;
-        sh.sum_hi = sh.sum_lo = 0;
-        sh.bad = sh.ovf = 0;
-    }
-    __syncthreads();
-
+    const int32_t tid = (int32_t)threadIdx.x, nthr = (int32_t)blockDim.x;
     const int32_t* __restrict__ Ag = bt.alloc_step + tv.lo;
     const int32_t* __restrict__ Fg = bt.free_step + tv.lo;
     const int64_t* __restrict__ Sg = bt.size_bytes + tv.lo;
     const int64_t* __restrict__ Og = offsets + tv.lo;
-    bool bad = false, ovf = false;
-    uint64_t sum = 0;
-    auto check = [&](int32_t a, int32_t f, int64_t sz, int64_t o) {
-        if (!tensor_ok(a, f, sz, T) || o < 0) {
-            bad = true;
-            return;
+    const bool vec = ((reinterpret_cast<uintptr_t>(Ag) | reinterpret_cast<uintptr_t>(Fg) |
+                       reinterpret_cast<uintptr_t>(Sg) | reinterpret_cast<uintptr_t>(Og)) & 15) == 0;
+    auto cidx = [&](int j) -> int32_t { return vec ? 4 * tid + j : tid + j * nthr; };
+    int32_t ca[kValCached], cf[kValCached];
+    int64_t cs[kValCached], co[kValCached];
+    if (vec && 4 * tid + 3 < n) {
+        const int4 a = __ldg(reinterpret_cast<const int4*>(Ag) + tid);
+        const int4 f = __ldg(reinterpret_cast<const int4*>(Fg) + tid);
+        const longlong2 s01 = __ldg(reinterpret_cast<const longlong2*>(Sg) + 2 * tid);
+        const longlong2 s23 = __ldg(reinterpret_cast<const longlong2*>(Sg) + 2 * tid + 1);
+        const longlong2 o01 = __ldg(reinterpret_cast<const longlong2*>(Og) + 2 * tid);
+        const longlong2 o23 = __ldg(reinterpret_cast<const longlong2*>(Og) + 2 * tid + 1);
+        ca[0] = a.x, ca[1] = a.y, ca[2] = a.z, ca[3] = a.w;
+        cf[0] = f.x, cf[1] = f.y, cf[2] = f.z, cf[3] = f.w;
+        cs[0] = s01.x, cs[1] = s01.y, cs[2] = s23.x, cs[3] = s23.y;
+        co[0] = o01.x, co[1] = o01.y, co[2] = o23.x, co[3] = o23.y;
+    } else {
+#pragma unroll
+        for (int j = 0; j < kValCached; ++j) {
+            const int32_t k = cidx(j);
+            ca[j] = cf[j] = 0;
+            cs[j] = co[j] = 0;
+            if (k < n) {
+                ca[j] = __ldg(Ag + k);
+                cf[j] = __ldg(Fg + k);
+                cs[j] = __ldg(Sg + k);
+                co[j] = __ldg(Og + k);
+            }
         }
-        sum = sat_add(sum, (uint64_t)sz);
-        if (o > INT64_MAX - sz) ovf = true;
-        atomicAdd(BEND + a, 1);
-    };
-    const bool vec_in = ((reinterpret_cast<uintptr_t>(Ag) | reinterpret_cast<uintptr_t>(Fg) |
-                          reinterpret_cast<uintptr_t>(Sg) | reinterpret_cast<uintptr_t>(Og)) & 15) == 0;
-    int k0 = 0;
-    if (vec_in) {
-        const int n4 = n >> 2;
-        for (int q = threadIdx.x; q < n4; q += blockDim.x) {
-            const int4 a = __ldg(reinterpret_cast<const int4*>(Ag) + q);
-            const int4 f = __ldg(reinterpret_cast<const int4*>(Fg) + q);
-            const longlong2 s01 = __ldg(reinterpret_cast<const longlong2*>(Sg) + 2 * q);
-            const longlong2 s23 = __ldg(reinterpret_cast<const longlong2*>(Sg) + 2 * q + 1);
-            const longlong2 o01 = __ldg(reinterpret_cast<const longlong2*>(Og) + 2 * q);
-            const longlong2 o23 = __ldg(reinterpret_cast<const longlong2*>(Og) + 2 * q + 1);
-            check(a.x, f.x, s01.x, o01.x);
-            check(a.y, f.y, s01.y, o01.y);
-            check(a.z, f.z, s23.x, o23.x);
-            check(a.w, f.w, s23.y, o23.y);
-        }
-        k0 = n4 << 2;
     }
-    for (int k = k0 + threadIdx.x; k < n; k += blockDim.x)
-        check(__ldg(Ag + k), __ldg(Fg + k), __ldg(Sg + k), __ldg(Og + k));
-    block_add_size_sum(sum, &sh.sum_hi, &sh.sum_lo);
-    if (bad) sh.bad = 1;
-    if (ovf) sh.ovf = 1;
+
+    const ValidateLayout L(kSmem ? n : bt.max_tensors, kSmem ? T : bt.max_steps);
+    unsigned char* base = kSmem ? smem_raw : ws + (size_t)b * ws_stride;
+    int2* FI = reinterpret_cast<int2*>(base + L.fi);
+    int32_t* BEND = reinterpret_cast<int32_t*>(base + L.bend);
+    if ((T & 3) == 0) {
+        for (int32_t t = tid; t < (T >> 2); t += nthr) reinterpret_cast<int4*>(BEND)[t] = make_int4(0, 0, 0, 0);
+    } else {
+        for (int32_t t = tid; t < T; t += nthr) BEND[t] = 0;
+    }
+    if (tid == 0) {
+        sh.key = ~0ull;
+        sh.sum[0] = sh.sum[1] = sh.sum[2] = 0;
+        sh.flags = 0;
+    }
     __syncthreads();
-    if (sh.bad || sh.ovf || size_sum_overflows(sh.sum_hi, sh.sum_lo)) {
-        if (threadIdx.x == 0) {
-            status[b] = sh.bad ? MP_EINVAL : MP_EOVERFLOW;
+
+    // Checks, flags and the alloc-step histogram.  The cached tensors keep
+    // their offset and end as 32-bit words from here on (all the narrow path
+    // needs); the wide path and the exact size sum read memory again.
+    int flags = 0;
+    auto take = [&](int32_t a, int32_t f, int64_t sz, int64_t o) -> uint64_t {
+        if (!tensor_ok(a, f, sz, T) || o < 0) {
+            flags |= kFlagInvalid;
+            return 0;
+        }
+        const uint64_t e = (uint64_t)o + (uint64_t)sz;  // both below 2^63: no wrap
+        flags |= (e >> 63) ? kFlagEndOvf : 0;
+        flags |= (e >> 32) ? kFlagWide : 0;
+        flags |= ((uint64_t)sz >> 32) ? kFlagBigSize : 0;
+        atomicAdd(BEND + a, 1);
+        return e;
+    };
+    uint32_t co32[kValCached], ce32[kValCached];
+#pragma unroll
+    for (int j = 0; j < kValCached; ++j) {
+        co32[j] = (uint32_t)co[j];
+        ce32[j] = cidx(j) < n ? (uint32_t)take(ca[j], cf[j], cs[j], co[j]) : 0u;
+    }
+    const int32_t nc = min(n, kValCached * nthr);
+    for (int32_t k = nc + tid; k < n; k += nthr) take(__ldg(Ag + k), __ldg(Fg + k), __ldg(Sg + k), __ldg(Og + k));
+    flags = (int)__reduce_or_sync(0xffffffffu, (unsigned)flags);
+    if ((tid & 31) == 0 && flags) atomicOr(&sh.flags, flags);
+    __syncthreads();
+    const int F = sh.flags;
+    bool sum_ovf = false;
+    if ((F & (kFlagInvalid | kFlagBigSize)) == kFlagBigSize) {  // the exact size sum (rare)
+        uint64_t sum = 0;
+        for (int32_t k = tid; k < n; k += nthr) sum = sat_add(sum, (uint64_t)__ldg(Sg + k));
+        block_add_size_limbs(sum, sh.sum);
+        __syncthreads();
+        sum_ovf = size_limbs_overflow(sh.sum);
+    }
+    if ((F & (kFlagInvalid | kFlagEndOvf)) || sum_ovf) {
+        if (tid == 0) {
+            status[b] = (F & kFlagInvalid) ? MP_EINVAL : MP_EOVERFLOW;
             verdict[b] = 0;
             if (conflict) conflict[2 * b] = conflict[2 * b + 1] = -1;
         }
@@ -117,33 +250,37 @@ k_validate(mp_batch bt, const int64_t* __restrict__ offsets, int32_t* __restrict
     }
     // Counting sort by alloc step: bucket starts, then scatter; afterwards
     // BEND[t] is the end of bucket t (tensors with alloc <= t).
-    block_excl_scan_array<int32_t, 8>(BEND, T, red);
-    for (int k = threadIdx.x; k < n; k += blockDim.x) {
-        const int32_t a = __ldg(Ag + k);
-        const int64_t o = __ldg(Og + k);
+    block_excl_scan_i32(BEND, T, red);
+    const bool wide = (F & kFlagWide) != 0;
+    uint2* REC32 = reinterpret_cast<uint2*>(base + L.rec);
+    longlong2* REC64 = reinterpret_cast<longlong2*>(base + L.rec);
+    auto scatter = [&](int32_t k, int32_t a, int32_t f, uint32_t o32, uint32_t e32) {
         const int32_t pos = atomicAdd(BEND + a, 1);
-        REC[pos] = make_longlong2(o, o + __ldg(Sg + k));
-        ID[pos] = k;
-        FP[pos] = __ldg(Fg + k);
+        if (wide) {
+            const int64_t o = __ldg(Og + k);
+            REC64[pos] = make_longlong2(o, o + __ldg(Sg + k));
+        } else {
+            REC32[pos] = make_uint2(o32, e32);
+        }
+        FI[pos] = make_int2(f, k);
+    };
+#pragma unroll
+    for (int j = 0; j < kValCached; ++j) {
+        const int32_t k = cidx(j);
+        if (k < n) scatter(k, ca[j], cf[j], co32[j], ce32[j]);
+    }
+    for (int32_t k = nc + tid; k < n; k += nthr) {
+        const uint32_t o32 = wide ? 0u : (uint32_t)__ldg(Og + k);
+        scatter(k, __ldg(Ag + k), __ldg(Fg + k), o32, wide ? 0u : o32 + (uint32_t)__ldg(Sg + k));
     }
     __syncthreads();
 
-    // Each overlapping pair once, from its earlier member in alloc order.
-    for (int p = threadIdx.x; p < n; p += blockDim.x) {
-        const int32_t stop = BEND[FP[p] - 1];
-        if (stop <= p + 1) continue;
-        const longlong2 ri = REC[p];
-        for (int q = p + 1; q < stop; ++q) {
-            const longlong2 rj = REC[q];
-            if (ri.x < rj.y && rj.x < ri.y) {
-                const uint32_t i = (uint32_t)ID[p], j = (uint32_t)ID[q];
-                const uint32_t lo = i < j ? i : j, hi = i < j ? j : i;
-                atomicMin(&sh.key, ((unsigned long long)lo << 32) | hi);
-            }
-        }
-    }
+    if (wide)
+        check_pairs(REC64, FI, BEND, n, &sh.key);
+    else
+        check_pairs(REC32, FI, BEND, n, &sh.key);
     __syncthreads();
-    if (threadIdx.x == 0) {
+    if (tid == 0) {
         const unsigned long long key = sh.key;
         const bool ok = key == ~0ull;
         verdict[b] = ok ? 1 : 0;

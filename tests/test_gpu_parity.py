@@ -123,6 +123,19 @@ def test_global_memory_path(cuda_lib, name, pol):
     assert_parity(ts, gpu_run(ts, name), oracle_run(ts, pol))
 
 
+def test_long_horizon_global_variants(cuda_lib):
+    """Traces of 40,000 steps: the profile's difference array no longer fits in
+    shared memory (it is built and scanned in the output slice itself) and the
+    validator's working set moves to the workspace; a short trace rides along."""
+    rng = np.random.default_rng(17)
+    T, n = 40000, 3000
+    a = rng.integers(0, T, size=n)
+    f = np.minimum(a + 1 + rng.geometric(0.01, size=n), T)
+    s = rng.integers(1, 1 << 24, size=n) * 64
+    ts = tg.from_arrays([(T, a, f, s), tg.config(0).trace(0), (T, a[:50], f[:50], s[:50] << 20)])
+    assert_parity(ts, gpu_run(ts, "first"), oracle_run(ts, oracle.FIT_FIRST))
+
+
 @pytest.mark.parametrize("name,pol", POLICIES)
 def test_long_lived_chain_workspace_path(cuda_lib, name, pol):
     """One component of 14,000 tensors that all live longer than 32 steps, on
@@ -197,6 +210,40 @@ def test_error_codes(cuda_lib):
         g, o = gpu_run(ts, name), oracle_run(ts, pol)
         assert o["st"][1].tolist() == [1, 1, 1, 1, 2, 1, 0]
         assert_parity(ts, g, o)
+
+
+def test_validator_error_codes(cuda_lib):
+    """The validator's own status codes: offsets past INT64_MAX - size, size sums past INT64_MAX,
+    negative offsets, and EINVAL winning over EOVERFLOW, each beside a valid trace."""
+    import paper_2203_00448_gb300 as mp
+
+    big = 2 ** 62
+    traces = [
+        (4, [(0, 2, 64), (1, 3, 64)]),                      # valid, no conflict
+        (4, [(0, 2, 64), (1, 3, 64)]),                      # end past INT64_MAX
+        (4, [(0, 1, big), (0, 2, big), (1, 3, 64)]),         # sizes sum past INT64_MAX
+        (4, [(0, 2, 64), (1, 3, 64)]),                      # negative offset
+        (4, [(0, 2, 64), (1, 3, 64), (2, 4, 64)]),          # end past INT64_MAX and an invalid offset
+        (4, [(0, 2, 64), (1, 3, 64)]),                      # address clash
+    ]
+    ts = tg.from_tuples(traces)
+    off = np.zeros(ts.n_tensors, dtype=np.int64)
+    tp = ts.trace_ptr
+    off[tp[0] + 1] = 64
+    off[tp[1] + 1] = 2 ** 63 - 1 - 32
+    off[tp[2] + 1] = 2 ** 62
+    off[tp[3] + 1] = -64
+    off[tp[4] + 1] = 2 ** 63 - 1
+    off[tp[4] + 2] = -1
+    off[tp[5] + 1] = 32
+    db = mp.DeviceBatch.from_host(ts, "cuda")
+    v, c, st = mp.validate_plan(db, torch.as_tensor(off, device="cuda"))
+    ov, oc, ost = oracle.validate_plan(ts, off)
+    assert ost.tolist() == [0, 2, 2, 1, 1, 0]
+    assert np.array_equal(st.cpu().numpy(), ost)
+    okm = ost == 0
+    assert np.array_equal(v.cpu().numpy()[okm], ov[okm]) and ov[okm].tolist() == [1, 0]
+    assert np.array_equal(c.cpu().numpy()[okm], oc[okm])
 
 
 def test_declared_bounds_and_csr_checked(cuda_lib):
