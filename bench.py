@@ -478,7 +478,7 @@ def run_gpu(args):
     # path, and D2H of every result, each step.
     e2e = None
     if not args.no_e2e:
-        hp = mp.HostPath(ts, dev, args.policy, stream=stream)
+        hp = mp.HostPath(ts, dev, args.policy, stream=stream, chunks=args.e2e_chunks)
         hp.stage(ts)
         for _ in range(max(1, args.warmup)):
             hp.run()
@@ -491,7 +491,8 @@ def run_gpu(args):
             hp.run()
         e2e_s = max_over_ranks((time.perf_counter() - t0) / e2e_steps, dist)
         e2e = {"value": total_tensors / e2e_s, "unit": UNIT, "h2d_bytes_per_step": hp.h2d_bytes,
-               "d2h_bytes_per_step": hp.d2h_bytes, "ms_per_step": 1e3 * e2e_s}
+               "d2h_bytes_per_step": hp.d2h_bytes, "ms_per_step": 1e3 * e2e_s,
+               "call": f"mp_plan_and_validate_host, {hp.chunks} chunks, pinned host buffers, host wall clock"}
 
     if rank != 0:
         if dist is not None:
@@ -639,6 +640,8 @@ def main(argv=None):
     ap.add_argument("--oracle-traces", type=int, default=4096,
                     help="traces of the workload the CPU-baseline leg runs through the oracle")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--e2e-chunks", type=int, default=4,
+                    help="runs of traces the end-to-end call pipelines its copies over")
     ap.add_argument("--no-breakdown", action="store_true",
                     help="skip the three-kernel breakdown (profiling runs that should launch the fused kernel only)")
     ap.add_argument("--traces", type=int, default=WORKLOAD["n_traces"],

@@ -170,6 +170,59 @@ mp_status mp_plan_and_validate(const mp_batch *batch, mp_fit_policy policy, int6
                                int64_t *offsets, int64_t *plan_peak, int32_t *verdict, int32_t *conflict,
                                int32_t *trace_status, void *workspace, size_t workspace_bytes, void *stream);
 
+/* Host buffers receiving the results of mp_plan_and_validate_host; the same
+ * arrays, sizes and meaning as the device outputs of mp_plan_and_validate.
+ * conflict may be NULL. */
+typedef struct mp_host_results {
+    int64_t *profile;      /* int64[n_steps] */
+    int64_t *peak_lb;      /* int64[B] */
+    int64_t *offsets;      /* int64[n_tensors] */
+    int64_t *plan_peak;    /* int64[B] */
+    int32_t *verdict;      /* int32[B] */
+    int32_t *conflict;     /* int32[2B], nullable */
+    int32_t *trace_status; /* int32[B] */
+} mp_host_results;
+
+/* Most chunks mp_plan_and_validate_host cuts a batch into. */
+#define MP_HOST_PATH_MAX_CHUNKS 64
+
+/* Bytes of device memory mp_plan_and_validate_host needs for this host batch
+ * cut into `chunks` pieces (inputs, outputs and planner workspace); 0 if the
+ * batch or chunk count is rejected. */
+size_t mp_host_path_bytes(const mp_batch *host_batch, int32_t chunks);
+
+/* The whole path (as mp_plan_and_validate: profile, greedy_by_size plan,
+ * validation) from HOST memory to HOST memory.  host_batch has the layout of
+ * mp_batch but every array pointer is a host pointer; its CSR arrays must
+ * start at 0, never decrease and end at n_tensors / n_steps (MP_EINVAL
+ * otherwise), and profile_ptr is required.  The batch is cut into at most
+ * `chunks` (0..MP_HOST_PATH_MAX_CHUNKS) runs of consecutive traces with about
+ * equal tensor counts; each run's inputs are copied to the device on
+ * copy_in_stream, planned on compute_stream once they have landed, and its
+ * profile and offsets copied back on copy_out_stream once planned, so the
+ * copies of both directions overlap the planning of other runs; the
+ * per-trace results follow the last run.  Page-locked (pinned) host memory
+ * is needed for the copies to overlap; pageable memory is correct but
+ * serialises them.  chunks = 0 stages nothing: the kernels read the inputs
+ * from, and write the results to, the host arrays themselves over the
+ * CPU-GPU link; every host array must then be page-locked memory mapped into
+ * the device's address space (cudaHostAlloc / cudaMallocHost, or
+ * cudaHostRegister with cudaHostRegisterMapped), else MP_EINVAL, and the
+ * device buffer holds only the planner's workspace.  device_buffer:
+ * caller-owned device memory of at least
+ * mp_host_path_bytes(host_batch, chunks) bytes, 256-byte aligned, holding the
+ * device copies and the workspace; not used concurrently by another call.
+ * The call only enqueues work: the host outputs are complete once
+ * copy_out_stream has reached its end (e.g. cudaStreamSynchronize), and the
+ * host inputs must stay unchanged until copy_in_stream has.  The three
+ * streams may be the same stream (no overlap).  Cross-stream order uses
+ * events the library creates once per device; concurrent callers on one
+ * device are serialised while they enqueue.  Return codes as for
+ * mp_plan_and_validate; per-trace errors in out->trace_status. */
+mp_status mp_plan_and_validate_host(const mp_batch *host_batch, mp_fit_policy policy, const mp_host_results *out,
+                                    int32_t chunks, void *device_buffer, size_t device_bytes, void *copy_in_stream,
+                                    void *compute_stream, void *copy_out_stream);
+
 /* Bytes of device workspace mp_validate_plan needs for this batch. */
 size_t mp_validate_workspace_bytes(const mp_batch *batch);
 

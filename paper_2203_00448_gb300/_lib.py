@@ -20,6 +20,8 @@ EXPORTS = (
     "mp_plan_greedy_by_size",
     "mp_plan_greedy_by_size_static",
     "mp_plan_and_validate",
+    "mp_host_path_bytes",
+    "mp_plan_and_validate_host",
     "mp_validate_workspace_bytes",
     "mp_validate_plan",
     "mp_peak",
@@ -56,6 +58,16 @@ class MpBatch(ctypes.Structure):
     ]
 
 
+class MpHostResults(ctypes.Structure):
+    """Mirror of struct mp_host_results."""
+
+    _fields_ = [(name, ctypes.c_void_p) for name in
+                ("profile", "peak_lb", "offsets", "plan_peak", "verdict", "conflict", "trace_status")]
+
+
+HOST_PATH_MAX_CHUNKS = 64
+
+
 class MemplanError(RuntimeError):
     def __init__(self, fn: str, status: int):
         super().__init__(f"{fn} returned {status_string(status)}")
@@ -86,6 +98,10 @@ def load(path: str = LIB_PATH):
     lib.mp_plan_greedy_by_size_static.restype = i32
     lib.mp_plan_and_validate.argtypes = [BP, i32, P, P, P, P, P, P, P, P, sz, P]
     lib.mp_plan_and_validate.restype = i32
+    lib.mp_host_path_bytes.argtypes = [BP, i32]
+    lib.mp_host_path_bytes.restype = sz
+    lib.mp_plan_and_validate_host.argtypes = [BP, i32, ctypes.POINTER(MpHostResults), i32, P, sz, P, P, P]
+    lib.mp_plan_and_validate_host.restype = i32
     lib.mp_validate_workspace_bytes.argtypes = [BP]
     lib.mp_validate_workspace_bytes.restype = sz
     lib.mp_validate_plan.argtypes = [BP, P, P, P, P, P, sz, P]

@@ -387,27 +387,25 @@ def _packed(specs, device=None, pin_memory=False):
 
 
 class HostPath:
-    """End-to-end use from host memory: copies a batch from pinned host memory
-    to the device, runs the whole path (one plan_and_validate call), and copies
-    every result back.
-
-    Inputs and outputs each live in one device buffer mirrored by one pinned
-    host buffer of the same layout, so a run is one copy in, the fused call
-    and one copy out.
+    """End-to-end use from host memory through mp_plan_and_validate_host: the
+    batch sits in pinned host buffers, and one call copies it to the device,
+    runs the whole path (profile, plan, validation) and copies every result
+    back, cut into `chunks` runs of traces so that the copies of both
+    directions overlap the planning of other runs (three streams).  With
+    ``chunks=0`` nothing is staged: the kernels read the pinned inputs and
+    write the pinned results directly over the CPU-GPU link.
 
     ``run(ts)`` takes a host batch (numpy arrays, e.g. tracegen.TraceSet) with
     the same shape as the one the object was built for and returns host
     numpy views of profile, peak_lb, offsets, plan_peak, verdict, conflict,
-    status.  All work is on the given (or current) stream; run() returns once
-    the results are on the host.
+    status; it returns once the results are on the host.
     """
 
     _IN = ("trace_ptr", "steps", "profile_ptr", "alloc_step", "free_step", "size_bytes")
     _OUT = ("profile", "peak_lb", "offsets", "plan_peak", "verdict", "conflict", "status")
 
-    def __init__(self, ts, device="cuda", policy="first", stream=None):
+    def __init__(self, ts, device="cuda", policy="first", stream=None, chunks: int = 4):
         self.policy = policy
-        self.stream = stream
         dev = torch.device(device)
         B, N, S = int(ts.n_traces), int(ts.n_tensors), int(ts.n_steps)
         in_specs = [("trace_ptr", (B + 1,), torch.int64), ("steps", (B,), torch.int32),
@@ -415,30 +413,32 @@ class HostPath:
                     ("free_step", (N,), torch.int32), ("size_bytes", (N,), torch.int64)]
         out_specs = [("profile", (S,), torch.int64), ("peak_lb", (B,), torch.int64), ("offsets", (N,), torch.int64),
                      ("plan_peak", (B,), torch.int64), ("verdict", (B,), torch.int32),
-                     ("conflict", (2 * B,), torch.int32), ("status", (1, B), torch.int32)]
-        self.dev_in, din = _packed(in_specs, dev)
+                     ("conflict", (2 * B,), torch.int32), ("status", (B,), torch.int32)]
         self.host_in_buf, self.host_in = _packed(in_specs, pin_memory=True)
-        self.dev_out, dout = _packed(out_specs, dev)
         self.host_out_buf, self.host_out = _packed(out_specs, pin_memory=True)
+        self._h2d = sum(int(self.host_in[k].numel()) * self.host_in[k].element_size() for k in self._IN)
+        self._d2h = sum(int(self.host_out[k].numel()) * self.host_out[k].element_size() for k in self._OUT)
         self.stage(ts)
-        self.dev_in.copy_(self.host_in_buf)
-        self.dev_batch = DeviceBatch(din["trace_ptr"], din["steps"], din["profile_ptr"], din["alloc_step"],
-                                     din["free_step"], din["size_bytes"], B, int(ts.max_tensors),
-                                     int(ts.max_steps), N, S)
-        buf = object.__new__(PathBuffers)
-        for k in self._OUT:
-            setattr(buf, k, dout[k])
-        buf.plan_ws, buf.validate_ws = Workspace(dev), Workspace(dev)
-        buf.plan_ws.get(plan_workspace_bytes(self.dev_batch))
-        self.buffers = buf
+        self.hb = _lib.MpBatch(B, int(ts.max_tensors), int(ts.max_steps), 0, N, S,
+                               *(self.host_in[k].data_ptr() for k in self._IN))
+        self.res = _lib.MpHostResults(*(self.host_out[k].data_ptr() for k in self._OUT))
+        self.chunks = max(0, min(int(chunks), _lib.HOST_PATH_MAX_CHUNKS))
+        need = int(_lib.load().mp_host_path_bytes(ctypes.byref(self.hb), self.chunks))
+        if need == 0 and B > 0:
+            raise MemplanError("mp_host_path_bytes", _lib.EINVAL)
+        self.dev_buf = torch.empty(max(need, 256), dtype=torch.uint8, device=dev)
+        with torch.cuda.device(dev):
+            self.compute_stream = stream or torch.cuda.current_stream(dev)
+            self.copy_in_stream = torch.cuda.Stream(dev)
+            self.copy_out_stream = torch.cuda.Stream(dev)
 
     @property
     def h2d_bytes(self) -> int:
-        return self.host_in_buf.numel()
+        return self._h2d
 
     @property
     def d2h_bytes(self) -> int:
-        return self.host_out_buf.numel()
+        return self._d2h
 
     def stage(self, ts):
         """Places a host batch into the pinned input buffer (host-side memcpy)."""
@@ -448,12 +448,13 @@ class HostPath:
     def run(self, ts=None):
         if ts is not None:
             self.stage(ts)
-        s = self.stream or torch.cuda.current_stream()
-        with torch.cuda.stream(s):
-            self.dev_in.copy_(self.host_in_buf, non_blocking=True)
-            plan_and_validate(self.dev_batch, self.policy, self.buffers, stream=s)
-            self.host_out_buf.copy_(self.dev_out, non_blocking=True)
-        s.synchronize()
-        out = {k: v.numpy() for k, v in self.host_out.items()}
-        out["status"] = out["status"][0]
-        return out
+        # the device buffer is reused: the previous call's compute must not
+        # overlap this call's copies (stream order covers the rest)
+        self.copy_in_stream.wait_stream(self.compute_stream)
+        _check("mp_plan_and_validate_host",
+               _lib.load().mp_plan_and_validate_host(
+                   ctypes.byref(self.hb), _policy(self.policy), ctypes.byref(self.res), self.chunks,
+                   self.dev_buf.data_ptr(), self.dev_buf.numel(), self.copy_in_stream.cuda_stream,
+                   self.compute_stream.cuda_stream, self.copy_out_stream.cuda_stream))
+        self.copy_out_stream.synchronize()
+        return {k: v.numpy() for k, v in self.host_out.items()}

@@ -124,3 +124,52 @@ def test_host_argument_errors_of_the_other_strategies(lib):
     for fn in ("mp_bump_workspace_bytes", "mp_breadth_workspace_bytes", "mp_replay_workspace_bytes"):
         assert getattr(lib, fn)(ctypes.byref(_batch())) == 0  # small traces: shared memory
         assert getattr(lib, fn)(ctypes.byref(big)) > 0
+
+
+def test_host_path_argument_errors(lib):
+    """mp_plan_and_validate_host checks its host batch, results, chunk count
+    and device buffer before any CUDA call (so this runs without a GPU)."""
+    import numpy as np
+
+    EINVAL, ENOMEM = _lib.EINVAL, _lib.ENOMEM
+    tp = np.array([0, 2, 2, 5], np.int64)
+    pp = np.array([0, 4, 4, 10], np.int64)
+    st = np.array([4, 0, 6], np.int32)
+    a = np.zeros(5, np.int32)
+    f = np.ones(5, np.int32)
+    s = np.full(5, 64, np.int64)
+
+    def hb(trace_ptr=tp, profile_ptr=pp):
+        return _lib.MpBatch(3, 3, 6, 0, 5, 10, trace_ptr.ctypes.data, st.ctypes.data, profile_ptr.ctypes.data,
+                            a.ctypes.data, f.ctypes.data, s.ctypes.data)
+
+    outs = [np.zeros(10, np.int64), np.zeros(3, np.int64), np.zeros(5, np.int64), np.zeros(3, np.int64),
+            np.zeros(3, np.int32), np.zeros(6, np.int32), np.zeros(3, np.int32)]
+    res = _lib.MpHostResults(*(o.ctypes.data for o in outs))
+    good = hb()
+    need = lib.mp_host_path_bytes(ctypes.byref(good), 2)
+    assert need > 0
+    assert lib.mp_host_path_bytes(ctypes.byref(good), 0) > 0  # the direct mode: workspace only
+    assert lib.mp_host_path_bytes(ctypes.byref(good), -1) == 0
+    assert lib.mp_host_path_bytes(ctypes.byref(good), _lib.HOST_PATH_MAX_CHUNKS + 1) == 0
+    D = 0x100000  # a fake device address: never dereferenced by a call that fails its checks
+
+    def call(b=good, policy=0, r=res, chunks=2, dbuf=D, dbytes=need):
+        return lib.mp_plan_and_validate_host(ctypes.byref(b), policy, ctypes.byref(r) if r is not None else None,
+                                             chunks, dbuf, dbytes, None, None, None)
+
+    for bad_tp in (np.array([1, 2, 2, 5], np.int64), np.array([0, 3, 2, 5], np.int64), np.array([0, 2, 2, 4], np.int64)):
+        assert call(b=hb(trace_ptr=bad_tp)) == EINVAL
+        assert lib.mp_host_path_bytes(ctypes.byref(hb(trace_ptr=bad_tp)), 2) == 0
+    assert call(b=hb(profile_ptr=np.array([0, 4, 4, 9], np.int64))) == EINVAL  # does not end at n_steps
+    assert call(policy=7) == EINVAL
+    assert call(r=None) == EINVAL
+    assert call(chunks=-1) == EINVAL
+    assert call(chunks=0, dbuf=None) == EINVAL
+    assert call(chunks=0, dbytes=0) == ENOMEM
+    assert call(dbuf=None) == EINVAL
+    assert call(dbuf=D + 8) == EINVAL  # not 256-byte aligned
+    assert call(dbytes=need - 1) == ENOMEM
+    bad_res = _lib.MpHostResults(*(o.ctypes.data for o in outs))
+    bad_res.offsets = outs[2].ctypes.data + 4  # misaligned int64 output
+    assert call(r=bad_res) == EINVAL

@@ -512,25 +512,30 @@ def test_replay_on_device_slabs(cuda_lib):
 # ------------------------------------------------------------- end to end from host memory
 
 def test_host_path_matches_the_device_path(cuda_lib):
-    """HostPath (one pinned buffer in, one out) gives the fused call's results,
-    also for a second batch of the same shape staged into the same buffers."""
+    """HostPath (mp_plan_and_validate_host: pinned host buffers, chunked copies
+    overlapping the planning, or none with the kernels reading and writing the
+    pinned buffers directly) gives the fused call's results for every chunk
+    count, also for a second batch of the same shape staged into the same
+    buffers, and with empty, failing and more-chunks-than-traces cases."""
     import paper_2203_00448_gb300 as mp
 
     cases = ((tg.config(2).select(range(0, 4096, 8)), tg.config(2).select(range(1, 4096, 8))),
-             (tg.random_small(41, 97, 120, 200, 1 << 30),))
+             (tg.random_small(41, 97, 120, 200, 1 << 30),),
+             (tg.from_tuples([(4, [(-1, 2, 8)]), (0, []), (6, [(0, 3, 64), (1, 4, 32), (3, 6, 8)]), (5, [])]),))
     for batches in cases:
-        hp = mp.HostPath(batches[0], "cuda", "first")
-        for ts in batches:
-            ref = fused_run(ts, "first")
-            out = hp.run(ts)
-            ok = ref["st"] == 0
-            assert np.array_equal(out["status"], ref["st"])
-            for k, ptr in (("offsets", ts.trace_ptr), ("profile", ts.profile_ptr)):
-                for b in np.nonzero(ok)[0]:
-                    assert np.array_equal(out[k][ptr[b]:ptr[b + 1]], ref[k][ptr[b]:ptr[b + 1]]), (k, b)
-            for k in ("peak_lb", "plan_peak", "verdict"):
-                assert np.array_equal(out[k][ok], ref[k][ok]), k
-            assert np.array_equal(out["conflict"].reshape(-1, 2)[ok], ref["conflict"][ok])
+        for chunks in (0, 1, 3, 8):
+            hp = mp.HostPath(batches[0], "cuda", "first", chunks=chunks)
+            for ts in batches:
+                ref = fused_run(ts, "first")
+                out = hp.run(ts)
+                ok = ref["st"] == 0
+                assert np.array_equal(out["status"], ref["st"])
+                for k, ptr in (("offsets", ts.trace_ptr), ("profile", ts.profile_ptr)):
+                    for b in np.nonzero(ok)[0]:
+                        assert np.array_equal(out[k][ptr[b]:ptr[b + 1]], ref[k][ptr[b]:ptr[b + 1]]), (k, b)
+                for k in ("peak_lb", "plan_peak", "verdict"):
+                    assert np.array_equal(out[k][ok], ref[k][ok]), k
+                assert np.array_equal(out["conflict"].reshape(-1, 2)[ok], ref["conflict"][ok])
 
 
 # ------------------------------------------------------------- greedy by breadth
