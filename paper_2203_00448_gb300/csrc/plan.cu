@@ -73,7 +73,7 @@ constexpr int32_t kLongStage = 2048; // CTA tier, data in the workspace: long-li
 constexpr long long kSpinCycles = 1ll << 31;  // a wait for another warp longer than this is a fault
 constexpr int32_t kValWide = 64;     // validation: windows longer than this get a warp each
 constexpr int32_t kFlowWarps = 16;   // warps that take members from a run's ready queue
-constexpr int32_t kDeferComp = 256;  // the 32-bit launch (data in shared memory) defers larger components
+constexpr int32_t kDeferComp = 1024;  // the 32-bit launch (data in shared memory) defers larger components
 constexpr int32_t kSpinPolls = 64;   // polls of a queue slot before the waiting warp starts to sleep between them
 constexpr int32_t kDeferred = -1;    // trace status between the two launches: needs 64-bit bytes
 
