@@ -20,7 +20,9 @@
  *   synchronising; outputs are valid once the stream reaches that point.
  * - The return value reports host-side problems only: MP_EINVAL for a NULL
  *   or misaligned pointer, a negative count or a too-small workspace;
- *   MP_ECUDA when a launch fails.  On any non-OK return nothing was enqueued.
+ *   MP_ECUDA when a launch fails.  After MP_EINVAL or MP_ENOMEM nothing was
+ *   enqueued; after MP_ECUDA (a failed launch, copy or event call) part of a
+ *   call's work may already be on its streams.
  * - Per-trace data errors are written to trace_status[b] on the device:
  *     MP_EINVAL    bad CSR range (trace_ptr not non-decreasing, beyond
  *                  n_tensors, or more than max_tensors tensors), T_b < 0 or
