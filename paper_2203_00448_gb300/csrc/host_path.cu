@@ -139,16 +139,14 @@ cudaError_t device_pool(EventPool** out) {
 // memory registered with CUDA, mapped into the device's address space);
 // nullptr if it cannot.
 template <typename T>
-T* device_view(const T* host, int64_t len, cudaError_t* err) {
+T* device_view(const T* host, int64_t len) {
     if (len <= 0) return nullptr;
     cudaPointerAttributes attr;
-    const cudaError_t e = cudaPointerGetAttributes(&attr, host);
-    if (e != cudaSuccess) {
+    if (cudaPointerGetAttributes(&attr, host) != cudaSuccess) {
         cudaGetLastError();  // an unregistered pointer: not an error of the context
         return nullptr;
     }
     if (attr.type != cudaMemoryTypeHost || attr.devicePointer == nullptr) return nullptr;
-    *err = cudaSuccess;
     return static_cast<T*>(attr.devicePointer);
 }
 
@@ -162,10 +160,9 @@ mp_status direct_path(const mp_batch& hb, mp_fit_policy policy, const mp_host_re
     if (device_buffer == nullptr || reinterpret_cast<uintptr_t>(device_buffer) % mp::kAlign != 0) return MP_EINVAL;
     if (device_bytes < std::max<size_t>(ws, mp::kAlign)) return MP_ENOMEM;
     if (B == 0) return MP_OK;
-    cudaError_t e = cudaSuccess;
     bool reachable = true;
     auto view = [&](auto* host, int64_t len) {
-        auto* d = device_view(host, len, &e);
+        auto* d = device_view(host, len);
         if (len > 0 && d == nullptr) reachable = false;
         return d;
     };
@@ -186,8 +183,8 @@ mp_status direct_path(const mp_batch& hb, mp_fit_policy policy, const mp_host_re
     if (!reachable) return MP_EINVAL;  // some host array is not mapped into the device's address space
     cudaStream_t s_run = static_cast<cudaStream_t>(compute_stream);
     cudaStream_t s_out = static_cast<cudaStream_t>(copy_out_stream);
-    e = mp::launch_plan_fused(dev, (int32_t)policy, profile, peak_lb, offsets, plan_peak, verdict, conflict, status,
-                              device_buffer, s_run);
+    cudaError_t e = mp::launch_plan_fused(dev, (int32_t)policy, profile, peak_lb, offsets, plan_peak, verdict,
+                                          conflict, status, device_buffer, s_run);
     if (e == cudaSuccess && s_out != s_run) {
         EventPool* pool = nullptr;
         e = device_pool(&pool);
