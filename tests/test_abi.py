@@ -173,3 +173,32 @@ def test_host_path_argument_errors(lib):
     bad_res = _lib.MpHostResults(*(o.ctypes.data for o in outs))
     bad_res.offsets = outs[2].ctypes.data + 4  # misaligned int64 output
     assert call(r=bad_res) == EINVAL
+
+
+def test_host_path_sizes_follow_the_chunking(lib):
+    """The host path's device buffer holds the batch, its results and the
+    planner workspace of the largest chunk: more chunks never need more, one
+    chunk needs the whole batch's workspace plus the copies, no chunking (0)
+    only that workspace, and an empty batch the same for any chunk count.
+    Host-only computation (no GPU)."""
+    import numpy as np
+
+    B, n, T = 64, 300, 400  # 300 tensors per trace: the CTA tier's per-trace buffers are sized
+    tp = np.arange(B + 1, dtype=np.int64) * n
+    pp = np.arange(B + 1, dtype=np.int64) * T
+    st = np.full(B, T, np.int32)
+    a = np.zeros(B * n, np.int32)
+    f = np.ones(B * n, np.int32)
+    s = np.full(B * n, 64, np.int64)
+    hb = _lib.MpBatch(B, n, T, 0, B * n, B * T, tp.ctypes.data, st.ctypes.data, pp.ctypes.data, a.ctypes.data,
+                      f.ctypes.data, s.ctypes.data)
+    sizes = [lib.mp_host_path_bytes(ctypes.byref(hb), k) for k in (1, 2, 4, 8, 64)]
+    assert all(x > 0 for x in sizes)
+    assert all(x >= y for x, y in zip(sizes, sizes[1:]))
+    inputs_outputs = (B * n) * 24 + (B * T) * 8  # alloc/free/size in, offsets and profile out
+    assert sizes[-1] >= inputs_outputs
+    direct = lib.mp_host_path_bytes(ctypes.byref(hb), 0)  # the whole batch's workspace, no copies
+    assert 0 < direct < sizes[0] and sizes[0] - direct >= inputs_outputs
+    tp0 = np.zeros(1, np.int64)
+    empty = _lib.MpBatch(0, 0, 0, 0, 0, 0, tp0.ctypes.data, 0, tp0.ctypes.data, 0, 0, 0)
+    assert lib.mp_host_path_bytes(ctypes.byref(empty), 4) == lib.mp_host_path_bytes(ctypes.byref(empty), 1)
