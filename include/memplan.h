@@ -54,7 +54,9 @@ typedef enum mp_status {
     MP_EINVAL = 1,
     MP_EOVERFLOW = 2,
     MP_ECUDA = 3,
-    MP_ETIMEOUT = 4, /* reserved for waits that give up; no entry point waits today */
+    MP_ETIMEOUT = 4, /* per-trace only: a wait of the planner on another warp or
+                        CTA gave up after its bound (see mp_plan_greedy_by_size);
+                        that trace's outputs are unspecified */
     MP_ENOMEM = 5,   /* workspace smaller than the matching *_workspace_bytes */
     MP_EINTERNAL = 6 /* per-trace only: a kernel found an inconsistency in its own
                         state (a library defect); that trace's outputs are unspecified */
@@ -109,7 +111,9 @@ mp_status mp_live_profile(const mp_batch *batch, int64_t *profile, int64_t *peak
                           int32_t *trace_status, void *stream);
 
 /* Bytes of device workspace mp_plan_greedy_by_size needs for this batch
- * (depends on the host scalars only).  0 means none. */
+ * (depends on the host scalars only).  0 means none; SIZE_MAX means the need
+ * does not fit in size_t (every call on such a batch returns MP_ENOMEM).
+ * Every *_workspace_bytes function below follows the same rule. */
 size_t mp_plan_workspace_bytes(const mp_batch *batch);
 
 /* greedy_by_size offset assignment (stage 2; Sec. 2.3, default strategy of
@@ -151,7 +155,10 @@ mp_status mp_plan_greedy_by_size(const mp_batch *batch, mp_fit_policy policy, in
  *   and must be serialised by the caller; the planner writes every scratch
  *   byte before reading it, so nothing needs clearing between calls;
  * - the array occupies device memory on every device that loads this library
- *   until the process exits.
+ *   until the process exits;
+ * - the looked-up address is kept for the life of the process: after
+ *   cudaDeviceReset on a device this entry point must not be called on that
+ *   device again (the array may then live at another address).
  * Other arguments and return codes as for mp_plan_greedy_by_size. */
 mp_status mp_plan_greedy_by_size_static(const mp_batch *batch, mp_fit_policy policy, int64_t *offsets,
                                         int64_t *plan_peak, int32_t *trace_status, void *stream);
@@ -190,7 +197,8 @@ typedef struct mp_host_results {
 
 /* Bytes of device memory mp_plan_and_validate_host needs for this host batch
  * cut into `chunks` pieces (inputs, outputs and planner workspace); 0 if the
- * batch or chunk count is rejected. */
+ * batch or chunk count is rejected, SIZE_MAX if the need does not fit in
+ * size_t. */
 size_t mp_host_path_bytes(const mp_batch *host_batch, int32_t chunks);
 
 /* The whole path (as mp_plan_and_validate: profile, greedy_by_size plan,
@@ -308,13 +316,27 @@ mp_status mp_plan_optimal(const mp_batch *batch, int64_t *offsets, int64_t *opt_
 /* Alignment of every trace's slab placed by mp_slab_layout. */
 #define MP_SLAB_ALIGN 256
 
-/* Places one slab per trace in a single device buffer (Sec. 3.3:
- * prim::AllocateSlab[total_size] per graph, every tensor a view at its
- * offset): slab_base[b] = sum over earlier traces of plan_peak rounded up to
- * MP_SLAB_ALIGN; slab_base[n_traces] = the buffer's size in bytes.
- * plan_peak: int64[n_traces] device (negative values count as 0; give failed
- * traces 0).  slab_base: int64[n_traces + 1] device.  One kernel. */
-mp_status mp_slab_layout(int32_t n_traces, const int64_t *plan_peak, int64_t *slab_base, void *stream);
+/* Places one slab per trace in a single device buffer and every tensor in it
+ * (Sec. 3.3: prim::AllocateSlab[total_size] per graph, every tensor a view
+ * prim::AllocateTensor[size, offset] into it).
+ * batch: n_traces is required; trace_ptr and n_tensors are read only when
+ *   tensor_addr is given (the other fields are not used).
+ * plan_peak: int64[n_traces] device, each trace's total_mem.
+ * trace_status: int32[n_traces] device or NULL; a trace whose status is not
+ *   MP_OK (a failed plan) gets an empty slab.  Negative peaks count as 0.
+ * slab_base: int64[n_traces + 1] device out: slab_base[b] = sum over earlier
+ *   traces of their slab rounded up to MP_SLAB_ALIGN; slab_base[n_traces] =
+ *   the buffer's size in bytes.
+ * offsets: int64[n_tensors] device, the plan (required with tensor_addr).
+ * tensor_addr: int64[n_tensors] device out or NULL: tensor_addr[i] =
+ *   slab_base[b] + offsets[i], the byte address of tensor i of trace b in the
+ *   buffer, or -1 for every tensor of a trace whose status is not MP_OK;
+ *   entries of a trace whose CSR range is unsound (as for trace_status
+ *   MP_EINVAL) and entries outside every trace are not written.
+ * Returns MP_EINVAL for a NULL or misaligned required array.  One kernel, two
+ * with tensor_addr. */
+mp_status mp_slab_layout(const mp_batch *batch, const int64_t *plan_peak, const int32_t *trace_status,
+                         const int64_t *offsets, int64_t *slab_base, int64_t *tensor_addr, void *stream);
 
 /* Bytes of device workspace mp_replay_plan needs for this batch. */
 size_t mp_replay_workspace_bytes(const mp_batch *batch);

@@ -12,8 +12,8 @@ and bump_allocation (the baseline strategy of Sec. 2.3), greedy by breadth
 Eq. 2.1 for traces of at most 10 tensors, and plans materialised on device
 slabs and replayed on real memory (Sec. 3.3).
 """
-from ._lib import (EINTERNAL, EINVAL, ENOMEM, EOVERFLOW, FIT_BEST, FIT_FIRST, OK, MemplanError,
-                   status_string)
+from ._lib import (EINTERNAL, EINVAL, ENOMEM, EOVERFLOW, ETIMEOUT, FIT_BEST, FIT_FIRST, OK, SLAB_ALIGN,
+                   MemplanError, status_string)
 from .api import (DeviceBatch, HostPath, PathBuffers, PathResult, Workspace, bump_workspace_bytes, live_profile,
                   materialize, peak, plan_and_validate, plan_bump, plan_greedy_by_breadth, plan_greedy_by_size,
                   plan_optimal,
@@ -25,5 +25,6 @@ __all__ = [
     "plan_and_validate", "plan_bump", "plan_greedy_by_breadth", "plan_greedy_by_size", "plan_optimal",
     "plan_workspace_bytes", "run_path",
     "materialize", "replay_plan", "slab_layout", "validate_plan", "validate_workspace_bytes", "MemplanError",
-    "status_string", "OK", "EINVAL", "EOVERFLOW", "ENOMEM", "EINTERNAL", "FIT_FIRST", "FIT_BEST",
+    "status_string", "OK", "EINVAL", "EOVERFLOW", "ENOMEM", "EINTERNAL", "ETIMEOUT", "FIT_FIRST", "FIT_BEST",
+    "SLAB_ALIGN",
 ]

@@ -66,6 +66,7 @@ class MpHostResults(ctypes.Structure):
 
 
 HOST_PATH_MAX_CHUNKS = 64
+SLAB_ALIGN = 256  # MP_SLAB_ALIGN
 
 
 class MemplanError(RuntimeError):
@@ -120,7 +121,7 @@ def load(path: str = LIB_PATH):
     lib.mp_breadth_workspace_bytes.restype = sz
     lib.mp_plan_greedy_by_breadth.argtypes = [BP, i32, P, P, P, P, sz, P]
     lib.mp_plan_greedy_by_breadth.restype = i32
-    lib.mp_slab_layout.argtypes = [i32, P, P, P]
+    lib.mp_slab_layout.argtypes = [BP, P, P, P, P, P, P]
     lib.mp_slab_layout.restype = i32
     lib.mp_replay_workspace_bytes.argtypes = [BP]
     lib.mp_replay_workspace_bytes.restype = sz

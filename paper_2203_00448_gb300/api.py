@@ -269,24 +269,28 @@ def slab_layout(plan_peak: torch.Tensor, plan_status: torch.Tensor | None = None
     prim::AllocateSlab per trace): int64[B + 1], the last entry the total.
     Traces whose plan_status is non-zero get an empty slab."""
     lib = _lib.load()
-    peaks = plan_peak if plan_status is None else torch.where(plan_status == 0, plan_peak, 0)
-    n = peaks.numel()
-    base = torch.empty(n + 1, dtype=torch.int64, device=peaks.device)
-    _check("mp_slab_layout", lib.mp_slab_layout(n, _ptr(peaks), base.data_ptr(), _stream_ptr(stream)))
+    n = plan_peak.numel()
+    base = torch.empty(n + 1, dtype=torch.int64, device=plan_peak.device)
+    s = _lib.MpBatch(n, 0, 0, 0, 0, 0, None, None, None, None, None, None)
+    _check("mp_slab_layout", lib.mp_slab_layout(ctypes.byref(s), _ptr(plan_peak), _ptr(plan_status), None,
+                                                base.data_ptr(), None, _stream_ptr(stream)))
     return base
 
 
 def materialize(batch: DeviceBatch, offsets: torch.Tensor, plan_peak: torch.Tensor,
                 plan_status: torch.Tensor | None = None, stream=None):
     """One device buffer holding every trace's slab, and every tensor's byte
-    address in it (Sec. 3.3's prim::AllocateTensor views): returns
-    (slab uint8 tensor, slab_base int64[B + 1], byte offset of each tensor in
-    the slab int64[n_tensors])."""
-    base = slab_layout(plan_peak, plan_status, stream)
+    address in it (Sec. 3.3's prim::AllocateTensor views; -1 for the tensors
+    of a failed trace): returns (slab uint8 tensor, slab_base int64[B + 1],
+    address of each tensor int64[n_tensors])."""
+    lib = _lib.load()
+    base = torch.empty(batch.n_traces + 1, dtype=torch.int64, device=batch.device)
+    where = _empty(batch.n_tensors, torch.int64, batch.device)
+    s = batch.struct()
+    _check("mp_slab_layout", lib.mp_slab_layout(ctypes.byref(s), _ptr(plan_peak), _ptr(plan_status), _ptr(offsets),
+                                                base.data_ptr(), _ptr(where), _stream_ptr(stream)))
     total = int(base[-1].item())
     slab = torch.empty(max(total, 1), dtype=torch.uint8, device=batch.device)
-    counts = batch.trace_ptr[1:] - batch.trace_ptr[:-1]
-    where = torch.repeat_interleave(base[:-1], counts) + offsets
     return slab, base, where
 
 

@@ -93,7 +93,7 @@ mp_status from_cuda(cudaError_t e) { return e == cudaSuccess ? MP_OK : MP_ECUDA;
 
 extern "C" {
 
-__attribute__((visibility("default"))) int32_t mp_abi_version(void) { return 1; }
+__attribute__((visibility("default"))) int32_t mp_abi_version(void) { return 2; }
 
 __attribute__((visibility("default"))) const char* mp_status_string(mp_status status) {
     switch (status) {
@@ -225,11 +225,21 @@ __attribute__((visibility("default"))) mp_status mp_plan_optimal(const mp_batch*
                                         static_cast<cudaStream_t>(stream)));
 }
 
-__attribute__((visibility("default"))) mp_status mp_slab_layout(int32_t n_traces, const int64_t* plan_peak,
-                                                                int64_t* slab_base, void* stream) {
-    if (n_traces < 0 || !array_ok(plan_peak, n_traces) || !array_ok(slab_base, (int64_t)n_traces + 1))
-        return MP_EINVAL;
-    return from_cuda(mp::launch_slab_layout(n_traces, plan_peak, slab_base, static_cast<cudaStream_t>(stream)));
+__attribute__((visibility("default"))) mp_status mp_slab_layout(const mp_batch* batch, const int64_t* plan_peak,
+                                                                const int32_t* trace_status, const int64_t* offsets,
+                                                                int64_t* slab_base, int64_t* tensor_addr,
+                                                                void* stream) {
+    if (batch == nullptr || batch->n_traces < 0 || batch->n_tensors < 0) return MP_EINVAL;
+    const int64_t B = batch->n_traces;
+    if (!array_ok(plan_peak, B) || !array_ok(slab_base, B + 1)) return MP_EINVAL;
+    if (trace_status != nullptr && !aligned(trace_status)) return MP_EINVAL;
+    if (tensor_addr != nullptr) {  // the per-tensor views need the CSR and the offsets
+        if (!array_ok(batch->trace_ptr, B ? B + 1 : 0) || !array_ok(offsets, batch->n_tensors) ||
+            !array_ok(tensor_addr, batch->n_tensors))
+            return MP_EINVAL;
+    }
+    return from_cuda(mp::launch_slab_layout(*batch, plan_peak, trace_status, offsets, slab_base, tensor_addr,
+                                            static_cast<cudaStream_t>(stream)));
 }
 
 __attribute__((visibility("default"))) size_t mp_replay_workspace_bytes(const mp_batch* batch) {

@@ -263,7 +263,7 @@ bool breadth_fits_smem(const mp_batch& bt) {
 
 size_t breadth_workspace_bytes(const mp_batch& bt) {
     if (bt.n_traces == 0 || breadth_fits_smem(bt)) return 0;
-    return (size_t)bt.n_traces * BreadthLayout(bt.max_tensors, bt.max_steps).total;
+    return mul_sat((size_t)bt.n_traces, BreadthLayout(bt.max_tensors, bt.max_steps).total);
 }
 
 cudaError_t launch_breadth(const mp_batch& bt, int32_t policy, int64_t* offsets, int64_t* plan_peak, int32_t* status,

@@ -130,7 +130,7 @@ bool bump_fits_smem(const mp_batch& bt) { return BumpLayout(bt.max_tensors, bt.m
 
 size_t bump_workspace_bytes(const mp_batch& bt) {
     if (bt.n_traces == 0 || bump_fits_smem(bt)) return 0;
-    return (size_t)bt.n_traces * BumpLayout(bt.max_tensors, bt.max_steps).total;
+    return mul_sat((size_t)bt.n_traces, BumpLayout(bt.max_tensors, bt.max_steps).total);
 }
 
 cudaError_t launch_bump(const mp_batch& bt, int64_t* offsets, int64_t* plan_peak, int32_t* status, void* workspace,

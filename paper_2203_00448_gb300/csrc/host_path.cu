@@ -32,24 +32,25 @@ HostPathLayout host_path_layout(const mp_batch& hb, size_t ws_bytes) {
     const size_t B = (size_t)hb.n_traces, N = (size_t)hb.n_tensors, S = (size_t)hb.n_steps;
     HostPathLayout L;
     size_t at = 0;
-    auto take = [&](size_t bytes) {
+    auto take = [&](size_t bytes) {  // saturates at SIZE_MAX: such a layout never fits a buffer
         const size_t here = at;
-        at += align_up(bytes);
+        at = bytes > SIZE_MAX - mp::kAlign ? SIZE_MAX : mp::add_sat(at, align_up(bytes));
         return here;
     };
-    L.trace_ptr = take((B + 1) * 8);
-    L.steps = take(B * 4);
-    L.profile_ptr = take((B + 1) * 8);
-    L.alloc = take(N * 4);
-    L.free_ = take(N * 4);
-    L.size = take(N * 8);
-    L.profile = take(S * 8);
-    L.offsets = take(N * 8);
-    L.peak_lb = take(B * 8);
-    L.plan_peak = take(B * 8);
-    L.verdict = take(B * 4);
-    L.conflict = take(B * 8);
-    L.status = take(B * 4);
+    using mp::mul_sat;
+    L.trace_ptr = take(mul_sat(B + 1, 8));
+    L.steps = take(mul_sat(B, 4));
+    L.profile_ptr = take(mul_sat(B + 1, 8));
+    L.alloc = take(mul_sat(N, 4));
+    L.free_ = take(mul_sat(N, 4));
+    L.size = take(mul_sat(N, 8));
+    L.profile = take(mul_sat(S, 8));
+    L.offsets = take(mul_sat(N, 8));
+    L.peak_lb = take(mul_sat(B, 8));
+    L.plan_peak = take(mul_sat(B, 8));
+    L.verdict = take(mul_sat(B, 4));
+    L.conflict = take(mul_sat(B, 8));
+    L.status = take(mul_sat(B, 4));
     L.workspace = take(ws_bytes);
     L.total = at;
     return L;

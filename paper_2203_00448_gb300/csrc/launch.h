@@ -39,6 +39,17 @@ cudaError_t max_resident_ctas(const void* func, int threads, size_t smem, int* c
 constexpr size_t kAlign = 256;
 __host__ __device__ constexpr size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
+// Workspace sizes saturate at SIZE_MAX instead of wrapping: a batch whose
+// need does not fit in size_t can then never pass a workspace-size check.
+inline size_t mul_sat(size_t a, size_t b) {
+    size_t r;
+    return __builtin_mul_overflow(a, b, &r) ? SIZE_MAX : r;
+}
+inline size_t add_sat(size_t a, size_t b) {
+    size_t r;
+    return __builtin_add_overflow(a, b, &r) ? SIZE_MAX : r;
+}
+
 cudaError_t launch_live_profile(const mp_batch& bt, int64_t* profile, int64_t* peak_lb, int32_t* status,
                                 cudaStream_t stream);
 
@@ -55,7 +66,8 @@ cudaError_t launch_optimal(const mp_batch& bt, int64_t* offsets, int64_t* opt_pe
                            cudaStream_t stream);
 
 size_t replay_workspace_bytes(const mp_batch& bt);
-cudaError_t launch_slab_layout(int32_t n_traces, const int64_t* plan_peak, int64_t* slab_base, cudaStream_t stream);
+cudaError_t launch_slab_layout(const mp_batch& bt, const int64_t* plan_peak, const int32_t* trace_status,
+                               const int64_t* offsets, int64_t* slab_base, int64_t* tensor_addr, cudaStream_t stream);
 cudaError_t launch_replay(const mp_batch& bt, const int64_t* offsets, const int64_t* slab_base, unsigned char* slab,
                           int64_t slab_bytes, int32_t* ok, int32_t* first_bad, int32_t* status, void* workspace,
                           cudaStream_t stream);

@@ -242,7 +242,8 @@ int32_t opt_chunks(const mp_batch& bt) {
 
 size_t optimal_workspace_bytes(const mp_batch& bt) {
     if (bt.n_traces == 0) return 0;
-    return align_up((size_t)bt.n_traces * (size_t)opt_chunks(bt) * sizeof(longlong2));
+    const size_t need = mul_sat(mul_sat((size_t)bt.n_traces, (size_t)opt_chunks(bt)), sizeof(longlong2));
+    return need > SIZE_MAX - kAlign ? SIZE_MAX : align_up(need);
 }
 
 cudaError_t launch_optimal(const mp_batch& bt, int64_t* offsets, int64_t* opt_peak, int32_t* status, void* workspace,

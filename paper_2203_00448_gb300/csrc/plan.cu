@@ -1577,9 +1577,9 @@ PlanWorkspace plan_workspace(const mp_batch& bt) {
         slices = std::max(slices, std::max(a.data_stride, b.data_stride));
     }
     const size_t cap2 = (size_t)pow2_at_least(bt.max_tensors > 0 ? bt.max_tensors : 1);
-    w.buf_offset = (size_t)bt.n_traces * slices;
+    w.buf_offset = mul_sat((size_t)bt.n_traces, slices);
     w.buf_stride = align_up(cap2 * 32);
-    w.total = bt.n_traces == 0 ? 0 : w.buf_offset + (size_t)bt.n_traces * w.buf_stride;
+    w.total = bt.n_traces == 0 ? 0 : add_sat(w.buf_offset, mul_sat((size_t)bt.n_traces, w.buf_stride));
     return w;
 }
 

@@ -16,7 +16,9 @@
 // the array's name as a device address, so the first call on each device
 // (made with that device current) looks the address up once with
 // cudaGetSymbolAddress and caches it; make that first call before any stream
-// capture.  Every call shares the one array: two calls whose kernels overlap
+// capture.  The cached address outlives a cudaDeviceReset, after which the
+// module may be loaded again elsewhere, so the entry point must not be used on
+// a device after it has been reset.  Every call shares the one array: two calls whose kernels overlap
 // on a GPU (different streams, or different host threads) race on it and
 // must be serialised by the caller.  The planner writes every scratch byte it
 // later reads, so nothing has to be cleared between calls.

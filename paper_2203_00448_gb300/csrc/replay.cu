@@ -175,19 +175,41 @@ k_replay(mp_batch bt, const int64_t* __restrict__ offsets, const int64_t* __rest
     }
 }
 
+// Slab of every trace: plan_peak rounded up to kAlign, 0 for a failed trace
+// (trace_status non-zero) or a negative peak; slab_base is their exclusive
+// scan, with the total after the last trace.
 __global__ void __launch_bounds__(1024) k_slab_layout(int32_t n_traces, const int64_t* __restrict__ plan_peak,
+                                                     const int32_t* __restrict__ trace_status,
                                                      int64_t* __restrict__ slab_base) {
     __shared__ int64_t red[40];
     int64_t carry = 0;
     for (int64_t base = 0; base < n_traces; base += blockDim.x) {
         const int64_t b = base + threadIdx.x;
-        const int64_t v = b < n_traces ? (int64_t)align_up((size_t)max(plan_peak[b], (int64_t)0)) : 0;
+        int64_t v = 0;
+        if (b < n_traces && (trace_status == nullptr || trace_status[b] == MP_OK))
+            v = (int64_t)align_up((size_t)max(plan_peak[b], (int64_t)0));
         int64_t tot;
         const int64_t pre = block_excl_scan<int64_t>(v, red, &tot) + carry;
         if (b < n_traces) slab_base[b] = pre;
         carry += tot;
     }
     if (threadIdx.x == 0) slab_base[n_traces] = carry;
+}
+
+// Byte address of every tensor in the slab buffer (Sec. 3.3's
+// prim::AllocateTensor[size, offset] view of prim::AllocateSlab): one CTA per
+// trace; slab_base[b] + offset for a trace with status 0 whose CSR range is
+// sound, -1 for the tensors of a failed trace.
+__global__ void __launch_bounds__(256) k_slab_addresses(mp_batch bt, const int64_t* __restrict__ offsets,
+                                                       const int32_t* __restrict__ trace_status,
+                                                       const int64_t* __restrict__ slab_base,
+                                                       int64_t* __restrict__ tensor_addr) {
+    const int b = blockIdx.x;
+    const int64_t lo = bt.trace_ptr[b], hi = bt.trace_ptr[b + 1];
+    if (lo < 0 || hi < lo || hi > bt.n_tensors) return;  // no sound range to write
+    const bool ok = trace_status == nullptr || trace_status[b] == MP_OK;
+    const int64_t sb = slab_base[b];
+    for (int64_t i = lo + threadIdx.x; i < hi; i += blockDim.x) tensor_addr[i] = ok ? sb + offsets[i] : -1;
 }
 
 bool replay_fits_smem(const mp_batch& bt) {
@@ -198,11 +220,15 @@ bool replay_fits_smem(const mp_batch& bt) {
 
 size_t replay_workspace_bytes(const mp_batch& bt) {
     if (bt.n_traces == 0 || replay_fits_smem(bt)) return 0;
-    return (size_t)bt.n_traces * ReplayLayout(bt.max_tensors, bt.max_steps).total;
+    return mul_sat((size_t)bt.n_traces, ReplayLayout(bt.max_tensors, bt.max_steps).total);
 }
 
-cudaError_t launch_slab_layout(int32_t n_traces, const int64_t* plan_peak, int64_t* slab_base, cudaStream_t stream) {
-    k_slab_layout<<<1, 1024, 0, stream>>>(n_traces, plan_peak, slab_base);
+cudaError_t launch_slab_layout(const mp_batch& bt, const int64_t* plan_peak, const int32_t* trace_status,
+                               const int64_t* offsets, int64_t* slab_base, int64_t* tensor_addr, cudaStream_t stream) {
+    k_slab_layout<<<1, 1024, 0, stream>>>(bt.n_traces, plan_peak, trace_status, slab_base);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess || tensor_addr == nullptr || bt.n_traces == 0) return e;
+    k_slab_addresses<<<(unsigned)bt.n_traces, 256, 0, stream>>>(bt, offsets, trace_status, slab_base, tensor_addr);
     return cudaGetLastError();
 }
 

@@ -339,7 +339,7 @@ static bool validate_fits_smem(const mp_batch& bt) {
 
 size_t validate_workspace_bytes(const mp_batch& bt) {
     if (bt.n_traces == 0 || validate_fits_smem(bt)) return 0;
-    return (size_t)bt.n_traces * ValidateLayout(bt.max_tensors, bt.max_steps).total;
+    return mul_sat((size_t)bt.n_traces, ValidateLayout(bt.max_tensors, bt.max_steps).total);
 }
 
 cudaError_t launch_validate(const mp_batch& bt, const int64_t* offsets, int32_t* verdict, int32_t* conflict,

@@ -41,7 +41,7 @@ def test_every_declared_symbol_exported(lib):
 
 
 def test_status_strings(lib):
-    assert lib.mp_abi_version() == 1
+    assert lib.mp_abi_version() == 2
     names = [lib.mp_status_string(k).decode() for k in range(7)]
     assert names == ["MP_OK", "MP_EINVAL", "MP_EOVERFLOW", "MP_ECUDA", "MP_ETIMEOUT", "MP_ENOMEM", "MP_EINTERNAL"]
     assert lib.mp_status_string(99).decode() == "MP_UNKNOWN"
@@ -115,8 +115,12 @@ def test_host_argument_errors_of_the_other_strategies(lib):
     assert need > 0
     assert lib.mp_plan_optimal(ctypes.byref(b), P, P, P, P, need - 1, None) == ENOMEM
     assert lib.mp_plan_optimal(ctypes.byref(b), P, P, P, None, need, None) == EINVAL
-    assert lib.mp_slab_layout(-1, P, P, None) == EINVAL
-    assert lib.mp_slab_layout(4, None, P, None) == EINVAL
+    assert lib.mp_slab_layout(None, P, None, None, P, None, None) == EINVAL
+    assert lib.mp_slab_layout(ctypes.byref(_batch(n_traces=-1)), P, None, None, P, None, None) == EINVAL
+    assert lib.mp_slab_layout(ctypes.byref(b), None, None, None, P, None, None) == EINVAL       # no peaks
+    assert lib.mp_slab_layout(ctypes.byref(b), P, P + 2, None, P, None, None) == EINVAL        # misaligned status
+    assert lib.mp_slab_layout(ctypes.byref(b), P, None, None, P, P, None) == EINVAL            # addresses, no plan
+    assert lib.mp_slab_layout(ctypes.byref(b), P, None, P, P, P + 4, None) == EINVAL           # misaligned addresses
     assert lib.mp_replay_plan(ctypes.byref(b), P, P, None, 64, P, P, P, None, 0, None) == EINVAL  # no slab
     assert lib.mp_replay_plan(ctypes.byref(b), P, P, P, -1, P, P, P, None, 0, None) == EINVAL     # negative size
     assert lib.mp_replay_plan(ctypes.byref(b), P, None, P, 64, P, P, P, None, 0, None) == EINVAL  # no slab bases
@@ -202,3 +206,20 @@ def test_host_path_sizes_follow_the_chunking(lib):
     tp0 = np.zeros(1, np.int64)
     empty = _lib.MpBatch(0, 0, 0, 0, 0, 0, tp0.ctypes.data, 0, tp0.ctypes.data, 0, 0, 0)
     assert lib.mp_host_path_bytes(ctypes.byref(empty), 4) == lib.mp_host_path_bytes(ctypes.byref(empty), 1)
+
+
+def test_workspace_sizes_saturate_instead_of_wrapping(lib):
+    """A batch whose planner workspace does not fit in size_t gets SIZE_MAX, so
+    no workspace (and not the fixed scratch of the no-allocation entry point)
+    can pass the size check; nothing is launched (fake device addresses)."""
+    P = 0x10000
+    size_max = (1 << 64) - 1
+    huge = _batch(n_traces=(1 << 31) - 1, max_tensors=(1 << 28) - 1, max_steps=(1 << 31) - 1)
+    assert lib.mp_plan_workspace_bytes(ctypes.byref(huge)) == size_max
+    for fn in ("mp_validate_workspace_bytes", "mp_bump_workspace_bytes", "mp_breadth_workspace_bytes",
+               "mp_replay_workspace_bytes"):
+        assert getattr(lib, fn)(ctypes.byref(huge)) == size_max, fn
+    assert lib.mp_plan_greedy_by_size(ctypes.byref(huge), 0, P, P, P, P, 1 << 40, None) == _lib.ENOMEM
+    assert lib.mp_plan_greedy_by_size_static(ctypes.byref(huge), 0, P, P, P, None) == _lib.ENOMEM
+    assert lib.mp_plan_and_validate(ctypes.byref(huge), 0, None, None, P, P, P, None, P, P, 1 << 40,
+                                    None) == _lib.ENOMEM

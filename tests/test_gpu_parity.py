@@ -464,14 +464,22 @@ def test_replay_on_device_slabs(cuda_lib):
                         [tg.config(2).trace(b) for b in range(0, 4096, 128)] +
                         [tg.random_small(31, 1, 60, 40, 1 << 12).trace(0), (3, [], [], [])])
     db = mp.DeviceBatch.from_host(ts, "cuda")
-    for plan in (lambda: mp.plan_greedy_by_size(db, "first"), lambda: mp.plan_greedy_by_size(db, "best"),
-                 lambda: mp.plan_bump(db)):
+    counts = np.diff(ts.trace_ptr)
+    for plan, ref in ((lambda: mp.plan_greedy_by_size(db, "first"), lambda: oracle.plan_greedy_by_size(ts, 0)),
+                      (lambda: mp.plan_greedy_by_size(db, "best"), lambda: oracle.plan_greedy_by_size(ts, 1)),
+                      (lambda: mp.plan_bump(db), lambda: oracle.plan_bump(ts))):
         off, pk, st = plan()
         slab, base, where = mp.materialize(db, off, pk, st)
         ok, first_bad, rst = mp.replay_plan(db, off, base, slab)
         torch.cuda.synchronize()
         assert bool((rst == 0).all()) and bool((ok == 1).all()) and bool((first_bad == -1).all())
         assert int(base[-1]) >= int(pk.sum())
+        # the library's tensor addresses: each trace's slab base plus the oracle's offset
+        o_off, o_pk, _ = ref()
+        hb = base.cpu().numpy()
+        sizes = (o_pk + mp.SLAB_ALIGN - 1) // mp.SLAB_ALIGN * mp.SLAB_ALIGN
+        assert np.array_equal(hb, np.concatenate([[0], np.cumsum(sizes)]))
+        assert np.array_equal(where.cpu().numpy(), np.repeat(hb[:-1], counts) + o_off)
 
     # planted clashes: in every other trace, one tensor moved onto a lifetime-overlapping one
     off, _, _ = mp.plan_greedy_by_size(db, "first")
@@ -485,6 +493,13 @@ def test_replay_on_device_slabs(cuda_lib):
             h[ts.trace_ptr[b] + j] = h[ts.trace_ptr[b] + i]
     bad_off = torch.from_numpy(h).cuda()
     pk2, st2 = mp.peak(db, bad_off)
+    # a failed trace gets an empty slab and address -1 for its tensors
+    fst = torch.zeros_like(st2)
+    fst[1] = oracle.EINVAL
+    _, fbase, fwhere = mp.materialize(db, bad_off, pk2, fst)
+    hb, hw = fbase.cpu().numpy(), fwhere.cpu().numpy()
+    assert hb[2] == hb[1] and (hw[ts.trace_ptr[1]:ts.trace_ptr[2]] == -1).all()
+    assert np.array_equal(hw[ts.trace_ptr[2]:], np.repeat(hb[2:-1], counts[2:]) + h[ts.trace_ptr[2]:])
     verdict, _, vst = mp.validate_plan(db, bad_off)
     slab, base, _ = mp.materialize(db, bad_off, pk2, st2)
     ok, first_bad, rst = mp.replay_plan(db, bad_off, base, slab)
