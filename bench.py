@@ -79,6 +79,33 @@ def dist_env():
     return int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)), int(os.environ.get("LOCAL_RANK", 0))
 
 
+def resolve_launch(gpus: int, env=None) -> str:
+    """How this process should honour --gpus N: "run" (the ranks already match:
+    one process for N = 1, or N torchrun ranks), "spawn" (N > 1 asked for
+    without torchrun: re-launch this command under torch.distributed.run with N
+    ranks) or "mismatch" (torchrun started a different number of ranks than
+    --gpus asks for: refuse rather than report the wrong n_gpus)."""
+    env = os.environ if env is None else env
+    if gpus < 1:
+        return "mismatch"
+    if "WORLD_SIZE" not in env:
+        return "run" if gpus == 1 else "spawn"
+    return "run" if int(env["WORLD_SIZE"]) == gpus else "mismatch"
+
+
+def spawn_ranks(gpus: int, argv) -> int:
+    """Re-runs this script under torch.distributed.run with one rank per GPU
+    (rendezvous on 127.0.0.1) and returns its exit status."""
+    import socket
+
+    with socket.socket() as sk:
+        sk.bind(("127.0.0.1", 0))
+        port = sk.getsockname()[1]
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", f"--nproc-per-node={gpus}",
+           "--master-addr", "127.0.0.1", "--master-port", str(port), os.path.abspath(__file__), *argv]
+    return subprocess.call(cmd)
+
+
 def shard_seed0(rank: int, n_traces: int = WORKLOAD["n_traces"]) -> int:
     """First seed of this rank's batch (weak scaling: every rank plans its own batch)."""
     return rank * n_traces
@@ -228,6 +255,18 @@ class ClockSampler:
                 self.samples.append((clk.value, mx.value, rs.value))
             time.sleep(0.001)
 
+    def sample_now(self):
+        """One reading from the calling thread (between timed steps)."""
+        if self.nvml is None:
+            return
+        import ctypes
+
+        lib, h, reasons = self.nvml
+        clk, mx, rs = ctypes.c_uint(), ctypes.c_uint(), ctypes.c_ulonglong()
+        if lib.nvmlDeviceGetClockInfo(h, 1, ctypes.byref(clk)) == 0 and \
+                lib.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx)) == 0 and reasons(h, ctypes.byref(rs)) == 0:
+            self.samples.append((clk.value, mx.value, rs.value))
+
     def __enter__(self):
         import threading
 
@@ -287,6 +326,39 @@ def oracle_baseline(ts, n_sample_traces: int):
     return sub.n_tensors / dt, dt, sub
 
 
+def _oracle_path_seconds(ts):
+    """Profile + plan (first fit) + validate of a TraceSet with the oracle; the seconds taken."""
+    import oracle
+
+    t0 = time.perf_counter()
+    oracle.live_profile(ts)
+    off, _, _ = oracle.plan_greedy_by_size(ts, oracle.FIT_FIRST)
+    oracle.validate_plan(ts, off)
+    return time.perf_counter() - t0
+
+
+def oracle_pool(cores: int):
+    """A spawn-started process pool for the all-cores oracle leg (spawned, so it
+    is safe whenever it is created; created before the first GPU call)."""
+    import multiprocessing as mproc
+
+    import tracegen
+
+    pool = mproc.get_context("spawn").Pool(cores)
+    pool.map(_oracle_path_seconds, [tracegen.random_small(1, 2, 4, 8)] * cores)  # workers up, oracle loaded
+    return pool
+
+
+def oracle_all_cores(ts, pool, cores: int):
+    """The oracle as it stands over the whole batch, its traces split into
+    `cores` interleaved parts run by `cores` processes at once; wall seconds."""
+    n_parts = min(cores, ts.n_traces)
+    parts = [ts.select(range(c, ts.n_traces, n_parts)) for c in range(n_parts)]
+    t0 = time.perf_counter()
+    pool.map(_oracle_path_seconds, parts)
+    return time.perf_counter() - t0, n_parts
+
+
 def run_reference(args):
     rank, world, _ = dist_env()
     if rank != 0:
@@ -321,9 +393,11 @@ def run_reference(args):
 # ----------------------------------------------------------------- GPU arm
 
 def run_gpu(args):
+    rank, world, local = dist_env()
+    cores = os.cpu_count() or 1
+    pool = oracle_pool(cores) if (rank == 0 and args.oracle_traces > 0 and world == 1) else None
     import torch
 
-    rank, world, local = dist_env()
     dist = None
     if world > 1:
         import torch.distributed as dist
@@ -387,11 +461,14 @@ def run_gpu(args):
         for k in range(args.steps):
             flush.zero_()
             step(events[k])
+            sampler.sample_now()  # between steps: the host is not inside any timed pair of events
         torch.cuda.synchronize()
         wall = time.perf_counter() - t0
     if dist is not None:
         dist.barrier()
-    step_ms = sum(ev[0].elapsed_time(ev[1]) for ev in events) / args.steps
+    step_times = [ev[0].elapsed_time(ev[1]) for ev in events]
+    step_ms = statistics.median(step_times)
+    step_ms_mean = statistics.fmean(step_times)
     step_ms_max = max_over_ranks(step_ms, dist)
     wall_max = max_over_ranks(wall, dist)
     total_tensors = sum_over_ranks(float(ts.n_tensors), dist)
@@ -523,23 +600,36 @@ def run_gpu(args):
             "algorithmic_bytes_per_launch": fused_bytes, "traffic": traffic}
     if args.oracle_traces > 0:
         ob_value, ob_dt, ob_sub = oracle_baseline(ts, args.oracle_traces)
-        cpu_baseline = {"value": ob_value, "unit": UNIT, "cores": 1, "kind": "oracle",
-                        "sample": f"first {ob_sub.n_traces} of {ts.n_traces} traces, profile + plan + validate, "
-                                  f"{ob_dt:.2f} s single-threaded"}
+        single = {"value": ob_value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                  "sample": f"first {ob_sub.n_traces} of {ts.n_traces} traces, profile + plan + validate, "
+                            f"{ob_dt:.2f} s single-threaded"}
+        if pool is not None:
+            wall_all, n_parts = oracle_all_cores(ob_sub, pool, cores)
+            cpu_baseline = {"value": ob_sub.n_tensors / wall_all, "unit": UNIT, "cores": n_parts, "kind": "oracle",
+                            "sample": f"first {ob_sub.n_traces} of {ts.n_traces} traces, profile + plan + validate, "
+                                      f"split over {n_parts} processes on {cores} host cores, {wall_all:.2f} s wall",
+                            "single_core": single}
+        else:
+            cpu_baseline = single
     else:
         cpu_baseline = None
+    if pool is not None:
+        pool.close()
+        pool.join()
     clocks = sampler.summary()
     issue = issue_roofline(ncu_record(FUSED, ts.n_tensors, "warp_inst"), step_ms * 1e-3,
                            torch.cuda.get_device_properties(dev).multi_processor_count,
                            clocks["sm_mhz"] or clocks["sm_max_mhz"])
     line = {
         "metric": METRIC, "value": total_tensors / (step_ms_max * 1e-3), "unit": UNIT, "n_gpus": world,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms_max, "higher_is_better": True,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms_max, "ms_per_step_mean": step_ms_mean,
+        "ms_per_step_min": min(step_times), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
         "config": {"workload": ts.name if world == 1 else WORKLOAD_NAME, "n_traces": ts.n_traces * world,
                    "tensors_per_trace": w["n"],
                    "steps_per_trace": w["T"], "policy": args.policy,
                    "l2": "flushed before every timed step (256 MiB device write outside the timed events)",
+                   "timing": f"median over ranks' median of {args.steps} event-timed steps",
                    "parallelism": f"dp{world} (traces sharded by rank, no collective)"},
         "validated_pairs_per_s": total_pairs / (step_ms_max * 1e-3),
         "wall_ms_per_step_incl_flush": 1e3 * wall_max / args.steps,
@@ -559,24 +649,11 @@ def run_gpu(args):
     return 0
 
 
-def _oracle_path(ts):
-    """Profile + plan (first fit) + validate of a TraceSet with the oracle; returns the seconds taken."""
-    import oracle
-
-    t0 = time.perf_counter()
-    oracle.live_profile(ts)
-    off, _, _ = oracle.plan_greedy_by_size(ts, oracle.FIT_FIRST)
-    oracle.validate_plan(ts, off)
-    return time.perf_counter() - t0
-
-
 def run_all_configs(args):
     """Every workload of tracegen.CONFIG_NAMES through one mp_plan_and_validate
     call, timed like the bench step, next to the oracle on 1 host core and on
     all host cores (traces split over processes).  One JSON line per workload;
     these are parity workloads with their own shapes, not the bench line."""
-    import multiprocessing as mproc
-
     import torch
 
     import paper_2203_00448_gb300 as mp
@@ -584,8 +661,7 @@ def run_all_configs(args):
     from paper_2203_00448_gb300 import build
 
     cores = os.cpu_count() or 1
-    pool = mproc.get_context("spawn").Pool(cores)  # before the first GPU call
-    pool.map(_oracle_path, [tracegen.random_small(1, 2, 4, 8)] * cores)  # workers up and the oracle loaded
+    pool = oracle_pool(cores)  # before the first GPU call
     build.build()
     dev = torch.device("cuda", torch.cuda.current_device())
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
@@ -609,12 +685,8 @@ def run_all_configs(args):
         ok = bool((buf.status[0] == 0).all()) and bool((buf.verdict == 1).all())
         ms = statistics.median(times)
         nbytes = algorithmic_bytes(FUSED, ts.n_tensors, ts.n_traces, ts.n_steps)
-        one_core = _oracle_path(ts)
-        n_chunks = min(cores, ts.n_traces)
-        chunks = [ts.select(range(c, ts.n_traces, n_chunks)) for c in range(n_chunks)]
-        t0 = time.perf_counter()
-        pool.map(_oracle_path, chunks)
-        all_cores = time.perf_counter() - t0
+        one_core = _oracle_path_seconds(ts)
+        all_cores, n_chunks = oracle_all_cores(ts, pool, cores)
         gbs = nbytes / (ms * 1e-3) / 1e9
         print(json.dumps({
             "workload": tracegen.CONFIG_NAMES[k], "policy": args.policy, "ok": ok, "n_traces": ts.n_traces,
@@ -653,6 +725,13 @@ def main(argv=None):
         return run_all_configs(args)
     if args.impl == "reference":
         return run_reference(args)
+    how = resolve_launch(args.gpus)
+    if how == "spawn":
+        return spawn_ranks(args.gpus, sys.argv[1:] if argv is None else list(argv))
+    if how == "mismatch":
+        print(json.dumps({"error": f"--gpus {args.gpus} but WORLD_SIZE={os.environ.get('WORLD_SIZE')}: launch one "
+                                   f"rank per GPU (torchrun --nproc-per-node {args.gpus}) or drop torchrun"}))
+        return 2
     return run_gpu(args)
 
 

@@ -30,6 +30,9 @@ def _worker(rank, world, port, out_dir):
     dist.init_process_group("gloo", rank=rank, world_size=world)
     r, w, _ = bench.dist_env()
     assert (r, w) == (rank, world)
+    # --gpus must match the ranks torchrun started: each rank refuses a mismatch
+    assert bench.resolve_launch(world) == "run"
+    assert bench.resolve_launch(world + 2) == "mismatch" and bench.resolve_launch(1) == "mismatch"
     n_traces = 6
     ts = tg.random_batch(bench.shard_seed0(r, n_traces), n_traces, 40, 64)
     off, pk, st = oracle.plan_greedy_by_size(ts, oracle.FIT_FIRST)
@@ -55,3 +58,18 @@ def test_two_rank_sharding_matches_single_process(tmp_path):
     assert all((p["st"] == 0).all() for p in parts)
     assert all(float(p["t_max"]) == 2.0 for p in parts)
     assert all(float(p["total"]) == whole.n_tensors for p in parts)
+
+
+def test_gpus_argument_without_torchrun():
+    """Outside torchrun, --gpus 1 runs in this process and --gpus N > 1 re-launches
+    the command with N ranks; a bad count is refused."""
+    import sys
+
+    sys.path.insert(0, os.path.dirname(os.path.dirname(os.path.abspath(__file__))))
+    import bench
+
+    assert bench.resolve_launch(1, {}) == "run"
+    assert bench.resolve_launch(4, {}) == "spawn"
+    assert bench.resolve_launch(0, {}) == "mismatch"
+    assert bench.resolve_launch(2, {"WORLD_SIZE": "2"}) == "run"
+    assert bench.resolve_launch(8, {"WORLD_SIZE": "2"}) == "mismatch"
