@@ -79,6 +79,21 @@ cudaError_t launch_breadth(const mp_batch& bt, int32_t policy, int64_t* offsets,
 cudaError_t launch_peak(const mp_batch& bt, const int64_t* offsets, int64_t* plan_peak, int32_t* status,
                         cudaStream_t stream);
 
+// Batches of at most kGridMaxTraces traces whose max_tensors exceeds
+// kGridMinTensors -- a few large traces -- are planned by the grid-wide
+// dataflow (grid.cu); every other batch by one CTA per trace (plan.cu).
+constexpr int32_t kGridMinTensors = 1024;
+constexpr int32_t kGridMaxTraces = 32;
+bool grid_path(const mp_batch& bt);
+size_t grid_workspace_bytes(const mp_batch& bt);
+// hold >= 0 is a test hook: the tensor with that slot id (trace * max_tensors
+// + alloc-order position) is never queued, so the bounded wait runs out.
+cudaError_t launch_grid_plan(const mp_batch& bt, int32_t policy, int64_t* offsets, int64_t* plan_peak,
+                             int32_t* status, void* workspace, int32_t hold, cudaStream_t stream);
+cudaError_t launch_grid_fused(const mp_batch& bt, int32_t policy, int64_t* profile, int64_t* peak_lb,
+                              int64_t* offsets, int64_t* plan_peak, int32_t* verdict, int32_t* conflict,
+                              int32_t* status, void* workspace, cudaStream_t stream);
+
 // Largest max_tensors mp_plan_greedy_by_size accepts (per-trace counts are
 // packed with a 2-bit tier tag into one int32).
 constexpr int32_t kPlanMaxTensors = (1 << 28) - 1;

@@ -991,45 +991,164 @@ __device__ __forceinline__ W block_excl_scan_w(W v, int64_t* red, W* total) {
     return block_excl_scan<W>(v, reinterpret_cast<W*>(red), total);
 }
 
-// Places the nx large components starting at LST[0, nx) with the whole CTA
-// (the 32-bit launch defers traces with components above kDeferComp, and
-// with its data in the workspace, every trace that needs this tier).  Each
-// is sorted into priority order; its long-lived members cut the order into
-// runs of short-lived ones, which the warps place together, each long-lived
-// one then by the whole CTA.  sort_smem: 2n entries of shared memory for
-// the sort when the data is there.  Returns this thread's largest end.
+// Places a component none of whose members lives longer than kLongLife
+// steps with one warp, in priority order 32 ranks at a time; ord: its members'
+// positions by rank.  Every member of a batch depends only on lower ranks:
+// those of earlier batches are final, and inside the batch the offsets are
+// found by rounds in which every lane recomputes its member's offset from the
+// current offsets of its predecessors (one snapshot per round).  The
+// dependencies are acyclic, so the system has one fixed point -- the
+// sequential definition's offsets -- and a round that changes nothing has
+// reached it; a member whose longest chain of predecessors inside the batch
+// has d links is final after round d, so at most 33 rounds are needed.  The
+// predecessors of a member are among the members of its window (allocated in
+// (a - lw, f)); up to 64 positions they are kept as a bit mask, else tested on
+// every pass.  Returns this lane's largest end; sets *fail to 2 if a batch does
+// not settle (an inconsistency, never expected).
+template <typename I, typename W>
+__device__ W place_comp_rounds(const ARec<I, W>* AR, W* OFFP, const int32_t* BEND, const int32_t* ord, int32_t p0,
+                               int32_t c, int32_t lw, int32_t policy, volatile int32_t* fail) {
+    const unsigned full = 0xffffffffu;
+    const int lane = threadIdx.x & 31;
+    volatile W* voff = OFFP;
+    W mx = 0;
+    for (int32_t r0 = 0; r0 < c; r0 += 32) {
+        const int32_t r = r0 + lane;
+        const bool act = r < c;
+        int32_t x = -1, w0 = 0, w1 = 0;
+        ARec<I, W> me{};
+        uint64_t pm = 0;
+        if (act) {
+            x = ord[r];
+            me = AR[x];
+            w0 = max(p0, (int32_t)me.a >= lw ? BEND[(int32_t)me.a - lw] : 0);
+            w1 = min(p0 + c, BEND[(int32_t)me.f - 1]);
+            if (w1 - w0 <= 64) {
+                for (int32_t q = w0; q < w1; ++q) {
+                    if (q == x) continue;
+                    const ARec<I, W> o = AR[q];
+                    if ((int32_t)o.a < (int32_t)me.f && (int32_t)me.a < (int32_t)o.f && precedes(o, me))
+                        pm |= 1ull << (q - w0);
+                }
+            }
+            voff[x] = 0;
+        }
+        const bool masked = w1 - w0 <= 64;
+        auto each = [&](auto&& fn) {
+            if (masked) {
+                for (uint64_t m = pm; m; m &= m - 1) {
+                    const int32_t q = w0 + __ffsll((long long)m) - 1;
+                    const W o = voff[q];
+                    fn(o, (W)(o + AR[q].s));
+                }
+            } else {
+                for (int32_t q = w0; q < w1; ++q) {
+                    if (q == x) continue;
+                    const ARec<I, W> oq = AR[q];
+                    if ((int32_t)oq.a < (int32_t)me.f && (int32_t)me.a < (int32_t)oq.f && precedes(oq, me)) {
+                        const W o = voff[q];
+                        fn(o, (W)(o + oq.s));
+                    }
+                }
+            }
+        };
+        __syncwarp();
+        W o = 0;
+        for (int round = 0;; ++round) {
+            W on = 0;
+            if (act) {
+                if (policy == MP_FIT_FIRST) {
+                    on = fit_first_scan<W>(me.s, each);
+                } else {
+                    W top = 0;
+                    each([&](W, W pe) { top = pe > top ? pe : top; });
+                    on = fit_best_scan<W>(me.s, top, each);
+                }
+            }
+            const bool changed = act && on != o;
+            __syncwarp();
+            if (act) voff[x] = on;
+            o = on;
+            __syncwarp();
+            if (!__any_sync(full, changed)) break;
+            if (round >= 40) {
+                *fail = 2;
+                break;
+            }
+        }
+        if (act) mx = o + me.s > mx ? o + me.s : mx;
+    }
+    return mx;
+}
+
+// Places the nx large components starting at LST[0, nx) (the 32-bit launch
+// defers traces with components above kDeferComp, and with its data in the
+// workspace, every trace that needs this tier).  Each is first sorted into
+// priority order by the whole CTA.  Components whose members all live at most
+// kLongLife steps are then placed concurrently, a warp each, by rounds
+// (place_comp_rounds).  In the others the long-lived members cut the priority
+// order into runs of short-lived ones, which the warps place together from a
+// ready queue, each long-lived one then by the whole CTA.  Returns this
+// thread's largest end.
 template <typename I, typename W, bool kSmem>
 __device__ __forceinline__ W large_tier(const ARec<I, W>* AR, W* OFFP, const int32_t* BEND, const uint32_t* SB,
-                                     const int32_t* NW, const int32_t* LST, int32_t nx, int32_t n, int32_t* sort_smem,
-                                     int32_t* ORD, int32_t* HR, int32_t* CNT, int32_t* QUE, int64_t* bo, int64_t* be,
+                                     const int32_t* NW, const int32_t* LST, int32_t nx, int32_t n, int32_t* ORD, int32_t* HR, int32_t* CNT, int32_t* QUE, int64_t* bo, int64_t* be,
                                      unsigned char* smem_raw, int32_t policy, int64_t* red, int32_t* s_cnt,
                                      int32_t* s_tail, int32_t* s_fail) {
-    const int warp = threadIdx.x >> 5;
+    const int warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
     W mx = 0;
     W* scratch = nullptr;
     const LongStage<W> st = long_stage<W>(smem_raw, &scratch);
+    // 1. every large component sorted into priority order: ORD[p0 + r] is the
+    // position of its member of rank r
     for (int32_t qc = 0; qc < nx; ++qc) {
         const int32_t p0 = LST[qc], sz = comp_size(SB, NW, p0, n);
         const int32_t len = (int32_t)pow2_at_least(sz);
-        // len entries: with the data in shared memory, the rp and ord regions
-        // together (2n entries); the ranks and the order below only overwrite
-        // entries already read
-        int32_t* sortbuf = kSmem ? sort_smem : ORD;
-        __syncthreads();  // the thread tier's RP is dead
+        // the sort buffer: with the data in shared memory the cnt and que
+        // regions (2n entries, len <= 2n; free until step 3), else the
+        // long-lived ranks' buffer (max_tensors rounded up to a power of two);
+        // neither overlaps ORD
+        int32_t* sortbuf = kSmem ? CNT : HR;
+        __syncthreads();  // the thread tier's RP, and the previous component's buffer, are dead
         for (int32_t x = threadIdx.x; x < len; x += blockDim.x) sortbuf[x] = x < sz ? p0 + x : -1;
         __syncthreads();
         block_bitonic_sort(sortbuf, len, [&](int32_t x, int32_t y) {  // sentinels (-1) sort last
             return y < 0 ? x >= 0 : (x >= 0 && precedes(AR[x], AR[y]));
         });
+        for (int32_t r = threadIdx.x; r < sz; r += blockDim.x) ORD[p0 + r] = sortbuf[r];
+    }
+    __syncthreads();
+    // 2. components without long-lived members: a warp each, all at once
+    for (int32_t qc = warp; qc < nx; qc += nwarps) {
+        const int32_t p0 = LST[qc], sz = comp_size(SB, NW, p0, n);
+        bool any_long = false;
+        uint32_t lw = 1;
+        for (int32_t k = (threadIdx.x & 31); k < sz; k += 32) {
+            const int32_t life = (int32_t)AR[p0 + k].f - (int32_t)AR[p0 + k].a;
+            any_long |= life > kLongLife;
+            if (life <= kLongLife) lw = max(lw, (uint32_t)life);
+        }
+        if (__any_sync(0xffffffffu, any_long)) continue;  // step 3
+        const W e = place_comp_rounds<I, W>(AR, OFFP, BEND, ORD + p0, p0, sz,
+                                            (int32_t)__reduce_max_sync(0xffffffffu, lw), policy, s_fail);
+        mx = max(mx, e);
+    }
+    __syncthreads();
+    // 3. components with long-lived members, one after the other: their
+    // long-lived members cut the priority order into runs of short-lived ones,
+    // which the warps place together, each long-lived one then by the whole CTA
+    for (int32_t qc = 0; qc < nx; ++qc) {
+        const int32_t p0 = LST[qc];
+        const int32_t sz = comp_size(SB, NW, p0, n);
+        const int32_t* ord = ORD + p0;
+        __syncthreads();
         int32_t nl = 0, lw = 1;
         for (int32_t r0 = 0; r0 < sz; r0 += blockDim.x) {
             const int32_t r = r0 + threadIdx.x;
             ARec<I, W> rx;
             int32_t flag = 0;
             if (r < sz) {
-                const int32_t px = sortbuf[r];
-                if constexpr (kSmem) ORD[r] = px;
-                rx = AR[px];
+                rx = AR[ord[r]];
                 const int32_t life = (int32_t)rx.f - (int32_t)rx.a;
                 flag = life > kLongLife ? 1 : 0;
                 if (!flag) lw = max(lw, life);
@@ -1047,6 +1166,7 @@ __device__ __forceinline__ W large_tier(const ARec<I, W>* AR, W* OFFP, const int
             }
             nl += tot;
         }
+        if (nl == 0) continue;  // placed in step 2 (nl is the block total: the same in every thread)
         __syncthreads();
         int64_t lw_max;
         block_excl_max((int64_t)lw, red, &lw_max);
@@ -1054,7 +1174,7 @@ __device__ __forceinline__ W large_tier(const ARec<I, W>* AR, W* OFFP, const int
         cp.AR = AR;
         cp.OFFP = OFFP;
         cp.BEND = BEND;
-        cp.ord = ORD;
+        cp.ord = ord;
         cp.hr = HR;
         cp.p0 = p0;
         cp.c = sz;
@@ -1433,7 +1553,7 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
     // ---- large components, the whole CTA each
     if (s_base[kBins] > s_base[kBinCta]) {
         const W e = large_tier<I, W, kSmem>(AR, OFFP, BEND, SB, NW, LST + s_base[kBinCta], s_base[kBins] - s_base[kBinCta],
-                                            n, kSmem ? reinterpret_cast<int32_t*>(base + L.rp) : nullptr, ORD, HR, CNT,
+                                            n, ORD, HR, CNT,
                                             QUE, bo, be, smem_raw, policy, red, &s_cnt, &s_tail, &s_fail);
         mx = max(mx, e);
     }
@@ -1501,7 +1621,7 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
                 out.conflict[2 * b + 1] = good ? -1 : (int32_t)(key & 0xffffffffu);
             }
         }
-        status[b] = s_fail ? MP_ETIMEOUT : MP_OK;
+        status[b] = s_fail == 2 ? MP_EINTERNAL : s_fail ? MP_ETIMEOUT : MP_OK;
     }
 }
 
@@ -1643,11 +1763,15 @@ cudaError_t launch_any(const mp_batch& bt, const PlanOut& out, void* workspace, 
 
 }  // namespace
 
-// One workspace size serves both the planner and the fused entry point.
-size_t plan_workspace_bytes(const mp_batch& bt) { return plan_workspace(bt).total; }
+// One workspace size serves both the planner and the fused entry point;
+// batches of large traces take the grid-wide dataflow (grid.cu).
+size_t plan_workspace_bytes(const mp_batch& bt) {
+    return grid_path(bt) ? grid_workspace_bytes(bt) : plan_workspace(bt).total;
+}
 
 cudaError_t launch_plan(const mp_batch& bt, int32_t policy, int64_t* offsets, int64_t* plan_peak,
                         int32_t* status, void* workspace, cudaStream_t stream) {
+    if (grid_path(bt)) return launch_grid_plan(bt, policy, offsets, plan_peak, status, workspace, -1, stream);
     const PlanOut out{policy, offsets, plan_peak, status, nullptr, nullptr, nullptr, nullptr};
     return launch_any<false>(bt, out, workspace, stream);
 }
@@ -1655,6 +1779,9 @@ cudaError_t launch_plan(const mp_batch& bt, int32_t policy, int64_t* offsets, in
 cudaError_t launch_plan_fused(const mp_batch& bt, int32_t policy, int64_t* profile, int64_t* peak_lb,
                               int64_t* offsets, int64_t* plan_peak, int32_t* verdict, int32_t* conflict,
                               int32_t* status, void* workspace, cudaStream_t stream) {
+    if (grid_path(bt))
+        return launch_grid_fused(bt, policy, profile, peak_lb, offsets, plan_peak, verdict, conflict, status,
+                                 workspace, stream);
     const PlanOut out{policy, offsets, plan_peak, status, profile, peak_lb, verdict, conflict};
     return launch_any<true>(bt, out, workspace, stream);
 }

@@ -138,7 +138,7 @@ __device__ __forceinline__ void check_pairs(const R* __restrict__ rec, const int
 // compares; the exact size sum is only formed when some size reaches 2^32
 // (below that, n < 2^31 sizes cannot sum past INT64_MAX).
 template <bool kSmem>
-__global__ void __launch_bounds__(kValidateThreads, kSmem ? 12 : 1)
+__global__ void __launch_bounds__(kValidateThreads, kSmem ? 9 : 1)
 k_validate(mp_batch bt, const int64_t* __restrict__ offsets, int32_t* __restrict__ verdict,
            int32_t* __restrict__ conflict, int32_t* __restrict__ status, unsigned char* __restrict__ ws,
            size_t ws_stride) {

@@ -178,6 +178,32 @@ def test_mid_size_component_workspace_path(cuda_lib, name, pol):
     assert_parity(ts, gpu_run(ts, name), oracle_run(ts, pol))
 
 
+@pytest.mark.parametrize("name,pol", POLICIES)
+def test_one_cta_per_trace_workspace_variants(cuda_lib, name, pol):
+    """Traces of at most 1,024 tensors over 60,000 steps: one CTA per trace,
+    with the working set in the workspace (too large for shared memory).  Sizes
+    summing below and above 2^32 take the 32-bit and the 64-bit launch; each
+    trace holds components of 33 to 700 tensors with long-lived members, so the
+    CTA tier runs on both."""
+    import paper_2203_00448_gb300 as mp
+
+    rng = np.random.default_rng(40)
+    T = 60000
+    traces = []
+    for n, scale in ((1000, 64), (1024, 1 << 26), (700, 4), (300, 1 << 30)):
+        a = np.sort(rng.integers(0, T - 400, size=n))
+        comp = rng.integers(0, 4, size=n) == 0  # a quarter of them crowd into one busy stretch
+        a[comp] = 20000 + rng.integers(0, 200, size=int(comp.sum()))
+        life = np.where(rng.random(n) < 0.1, rng.integers(33, 300, size=n), rng.integers(1, 6, size=n))
+        f = np.minimum(a + life, T)
+        s = rng.integers(1, 1 << 10, size=n) * scale
+        traces.append((T, a, f, s))
+    ts = tg.from_arrays(traces)
+    db = mp.DeviceBatch.from_host(ts, "cuda")
+    assert ts.max_tensors <= 1024 and mp.plan_workspace_bytes(db) > 0
+    assert_parity(ts, gpu_run(ts, name), oracle_run(ts, pol))
+
+
 def test_empty_and_degenerate(cuda_lib):
     ts = tg.from_tuples([(0, []), (5, []), (1, [(0, 1, 1)]), (3, [(0, 3, 7), (0, 3, 7), (1, 2, 7)]),
                          (4, [(0, 4, 2 ** 40), (0, 4, 2 ** 40)])])
