@@ -24,7 +24,7 @@ cudaError_t set_smem_limit(const void* func, size_t bytes) {
     if (e != cudaSuccess) return e;
     std::lock_guard<std::mutex> lock(mu);
     if (done.count({dev, func})) return cudaSuccess;
-    e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemCeiling);
+    e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)std::max(bytes, kSmemCeiling));
     if (e == cudaSuccess) done.insert({dev, func});
     return e;
 }

@@ -66,9 +66,23 @@ constexpr int kGridWarps = kGridThreads / 32;
 constexpr int kPrepThreads = 512;
 constexpr int kFinishThreads = 256;
 constexpr int32_t kGridLong = 32;             // lives above this many steps: long-lived, placed by a CTA
-constexpr size_t kGridSmem = 192 * 1024;      // flow CTA: one region of (offset, end) pairs
-constexpr int32_t kRegionPairs = (int32_t)(kGridSmem / 16);
-constexpr int32_t kWarpPairs = 512;  // predecessors a warp holds while it places a short tensor
+// Flow CTA shared memory: a region for the item being placed, then a cache of
+// the batch's long-lived records.  A CTA item uses the region for up to
+// kLongPredPairs predecessor pairs and kLongSuccs successor slots; a warp item
+// uses its warp's 1/16 of it for up to kWarpSortPairs pairs (kWarpPairs
+// predecessors, padded for the sort) and kWarpSuccs successor slots.
+constexpr size_t kRegionBytes = 176 * 1024;
+constexpr int32_t kLongCache = 2400;          // long-lived records cached per CTA (20 bytes each)
+constexpr size_t kCacheBytes = (size_t)kLongCache * 20;
+constexpr size_t kGridSmem = kRegionBytes + kCacheBytes;
+constexpr int32_t kLongPredPairs = 9216;
+constexpr int32_t kLongSuccs = (int32_t)((kRegionBytes - (size_t)kLongPredPairs * 16) / 4);
+constexpr int32_t kRegionPairs = kLongPredPairs;  // CTA-item pairs beyond this go to the overflow buffer
+constexpr int32_t kWarpBytes = (int32_t)(kRegionBytes / 16);
+constexpr int32_t kWarpSortPairs = 512;
+constexpr int32_t kWarpPairs = 448;  // predecessors a warp holds while it places a short tensor
+constexpr int32_t kWarpSuccs = (kWarpBytes - kWarpSortPairs * 16) / 4;
+static_assert(kLongSuccs >= 1024 && kWarpSuccs >= 512, "successor lists");
 constexpr int kMaxLongCtas = 32;              // CTAs that place CTA items (and own an overflow buffer)
 constexpr int32_t kGridValWide = 64;          // validation windows longer than this: a warp each
 #ifdef MP_TEST_GRID_SPIN_CYCLES
@@ -131,6 +145,19 @@ struct GridOut {
     int64_t* peak_lb;
     int32_t* verdict;
     int32_t* conflict;
+};
+
+// The long-lived records of the batch, trace after trace in long-list order,
+// in a CTA's shared memory (when they fit): size, alloc and free step, and
+// alloc-order position.  base[b] is where trace b's start (32 traces at most).
+struct LongCache {
+    int64_t* s;
+    int32_t* a;
+    int32_t* f;
+    int32_t* q;
+    const int32_t* base;  // null: no cache, read the long list from global memory
+    const int32_t* lw;    // per trace: the longest short life (always set)
+    const int32_t* nl;    // per trace: the number of long-lived records (always set)
 };
 
 // ---------------------------------------------------------------- memory order
@@ -203,12 +230,12 @@ __device__ __forceinline__ GRec load_rec(const GridWs& w, int64_t g) {
 struct Cands {
     int32_t w0, w1, nlong;
 };
-__device__ __forceinline__ Cands cands_of(const GridWs& w, const TraceInfo& ti, const Node& x) {
+__device__ __forceinline__ Cands cands_of(const GridWs& w, int32_t lw, int32_t nlong, const Node& x) {
     const int32_t* bend = w.bend + (int64_t)x.b * w.TS;
     Cands c;
-    c.w0 = x.r.a >= ti.lw ? __ldg(bend + (x.r.a - ti.lw)) : 0;
+    c.w0 = x.r.a >= lw ? __ldg(bend + (x.r.a - lw)) : 0;
     c.w1 = __ldg(bend + (x.r.f - 1));
-    c.nlong = ti.nlong;
+    c.nlong = nlong;
     return c;
 }
 
@@ -219,14 +246,25 @@ struct Cand {
 };
 
 // Loads candidate k of x's sets -- window positions first (short-lived
-// records only), then long-list entries -- and returns whether it overlaps x
-// in lifetime (x itself and long-lived records met in the window do not).
-__device__ __forceinline__ bool fetch_cand(const GridWs& w, const Node& x, const Cands& c, int32_t k, Cand* cd) {
+// records only), then long-list entries (from the CTA's cache when there is
+// one) -- and returns whether it overlaps x in lifetime (x itself and
+// long-lived records met in the window do not).
+__device__ __forceinline__ bool fetch_cand(const GridWs& w, const LongCache& lc, const Node& x, const Cands& c,
+                                           int32_t k, Cand* cd) {
     const int32_t nwin = c.w1 - c.w0;
     int32_t q;
     if (k < nwin) {
         q = c.w0 + k;
     } else if (k < nwin + c.nlong) {
+        if (lc.base) {
+            const int32_t i = lc.base[x.b] + (k - nwin);
+            q = lc.q[i];
+            cd->slot = x.base + q;
+            cd->r.s = lc.s[i];
+            cd->r.a = lc.a[i];
+            cd->r.f = lc.f[i];
+            return q != x.p && overlaps(cd->r, x.r);
+        }
         q = __ldg(w.ll + x.base + (k - nwin));
     } else {
         cd->r.a = INT32_MAX;  // past the sets
@@ -376,10 +414,11 @@ __global__ void __launch_bounds__(kPrepThreads) k_grid_prep(mp_batch bt, GridOut
 // ---------------------------------------------------------------- flow
 
 constexpr int kU = 2;  // candidates per lane whose loads are in flight together
-constexpr int32_t kWarpSuccs = 1024;  // successors a warp lists while it places a short tensor
 
 // Gap search of a warp over predecessor pairs supplied by each(fn), which
-// calls fn(off, end) for every pair held by the calling lane.
+// calls fn(off, end) for every pair held by the calling lane: FIRST jumps to
+// the largest conflicting end until nothing conflicts; BEST walks the free
+// holes below the top.
 template <typename Each>
 __device__ int64_t warp_fit(int64_t s, int32_t policy, Each&& each) {
     if (policy == MP_FIT_FIRST) {
@@ -424,12 +463,70 @@ __device__ int64_t warp_fit(int64_t s, int32_t policy, Each&& each) {
     return best;
 }
 
+// Gap search of a warp over np <= kWarpSortPairs pairs in buf: a bitonic sort
+// by offset, then one scan in which the gap before pair k is its offset minus
+// the largest end before it (FIRST: the lowest gap that fits; BEST: the
+// smallest, the lowest on ties; none: the largest end).
+__device__ int64_t warp_sorted_fit(int64_t s, int32_t policy, int64_t* buf, int32_t np) {
+    const int lane = threadIdx.x & 31;
+    const unsigned full = 0xffffffffu;
+    int32_t plen = 1;
+    while (plen < np) plen <<= 1;
+    for (int32_t k = np + lane; k < plen; k += 32) buf[2 * k] = buf[2 * k + 1] = INT64_MAX;
+    __syncwarp();
+    for (int32_t kk = 2; kk <= plen; kk <<= 1) {
+        for (int32_t j = kk >> 1; j > 0; j >>= 1) {
+            for (int32_t t = lane; t < (plen >> 1); t += 32) {
+                const int32_t lo = 2 * t - (t & (j - 1)), hi = lo + j;
+                const bool up = (lo & kk) == 0;
+                const int64_t xo = buf[2 * lo], yo = buf[2 * hi];
+                if (up ? yo < xo : xo < yo) {
+                    const int64_t xe = buf[2 * lo + 1];
+                    buf[2 * lo] = yo;
+                    buf[2 * hi] = xo;
+                    buf[2 * lo + 1] = buf[2 * hi + 1];
+                    buf[2 * hi + 1] = xe;
+                }
+            }
+            __syncwarp();
+        }
+    }
+    const int32_t chunk = (np + 31) / 32;
+    const int32_t k0 = min(np, lane * chunk), k1 = min(np, k0 + chunk);
+    int64_t local = 0;
+    for (int32_t k = k0; k < k1; ++k) local = max(local, buf[2 * k + 1]);
+    int64_t incl = local;  // inclusive prefix max of the lanes' chunk maxima
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int64_t u = __shfl_up_sync(full, incl, o);
+        if (lane >= o) incl = u > incl ? u : incl;
+    }
+    const int64_t top = __shfl_sync(full, incl, 31);
+    int64_t prev = __shfl_up_sync(full, incl, 1);
+    if (lane == 0) prev = 0;
+    int64_t key = INT64_MAX, val = INT64_MAX;
+    for (int32_t k = k0; k < k1; ++k) {
+        const int64_t gl = buf[2 * k] - prev;
+        if (gl >= s) {
+            const int64_t kx = policy == MP_FIT_FIRST ? prev : gl;  // prev grows with k
+            if (kx < key || (kx == key && prev < val)) {
+                key = kx;
+                val = prev;
+            }
+        }
+        prev = max(prev, buf[2 * k + 1]);
+    }
+    warp_min_pair(key, val);
+    return key == INT64_MAX ? top : val;
+}
+
 // Visits x's candidates with one warp, kU per lane with their loads in
 // flight together: fn(hit, cand) on every lane in warp-uniform rounds, hit
 // meaning the candidate overlaps x.  The long list (ascending alloc steps)
 // stops after a round in which every candidate starts at or after f_x.
 template <typename Fn>
-__device__ __forceinline__ void warp_visit(const GridWs& w, const Node& x, const Cands& c, Fn&& fn) {
+__device__ __forceinline__ void warp_visit(const GridWs& w, const LongCache& lc, const Node& x, const Cands& c,
+                                           Fn&& fn) {
     const int lane = threadIdx.x & 31;
     const int32_t nwin = c.w1 - c.w0, ncand = nwin + c.nlong;
     for (int32_t k0 = 0; k0 < ncand; k0 += 32 * kU) {
@@ -439,7 +536,7 @@ __device__ __forceinline__ void warp_visit(const GridWs& w, const Node& x, const
 #pragma unroll
         for (int u = 0; u < kU; ++u) {
             const int32_t k = k0 + u * 32 + lane;
-            hit[u] = fetch_cand(w, x, c, k, &cd[u]);
+            hit[u] = fetch_cand(w, lc, x, c, k, &cd[u]);
             past &= k < nwin ? false : cd[u].r.a >= x.r.f;
         }
 #pragma unroll
@@ -448,28 +545,42 @@ __device__ __forceinline__ void warp_visit(const GridWs& w, const Node& x, const
     }
 }
 
+// Drops the count of a successor of a placed tensor; returns true if it
+// became ready.  The caller either queues it or, as a continuation, places it
+// next itself.
+__device__ __forceinline__ bool drop(const GridWs& w, int64_t slot) { return atomicSub(w.cnt + slot, 1) == 1; }
+
+// The class of a tensor that became ready (read after the acquiring fence).
+__device__ __forceinline__ bool cta_item(const GridWs& w, int64_t slot) {
+    __threadfence();
+    return __ldcg(w.cls + slot) != 0;
+}
+
 // A short-lived tensor with at most kWarpPairs predecessors, placed by one
-// warp.  buf: the warp's share of the region -- kWarpPairs (offset, end) pairs,
-// then kWarpSuccs successor slots.  One pass over the candidates gathers the
-// predecessors and lists the successors; after the offset is published the
-// successors' counts drop.
-__device__ void place_short(const GridWs& w, int64_t g, int32_t policy, int64_t* buf) {
+// warp.  buf: the warp's share of the region -- kWarpSortPairs (offset, end)
+// pairs, then kWarpSuccs successor slots.  One pass over the candidates
+// gathers the predecessors and lists the successors; the gap search runs on
+// the gathered pairs (BEST with many of them sorts them first); after the
+// offset is published the successors' counts drop.  Returns a successor that
+// became ready and is a warp item, for this warp to place next (-1 if none);
+// the other ready ones are queued.
+__device__ int64_t place_short(const GridWs& w, const LongCache& lc, int64_t g, int32_t policy, int64_t* buf) {
     const int lane = threadIdx.x & 31;
     const unsigned full = 0xffffffffu, lt = (1u << lane) - 1u;
     const Node x = load_node(w, g);
-    const TraceInfo ti = w.ti[x.b];
-    const Cands c = cands_of(w, ti, x);
-    int32_t* sbuf = reinterpret_cast<int32_t*>(buf + 2 * kWarpPairs);
+    const Cands c = cands_of(w, lc.lw[x.b], lc.nl[x.b], x);
+    int32_t* sbuf = reinterpret_cast<int32_t*>(buf + 2 * kWarpSortPairs);
+    // the predecessors' (slot, size), then all their offsets at once: one
+    // round trip to L2 instead of one per round of candidates
     int32_t np = 0, ns = 0;
-    warp_visit(w, x, c, [&](bool hit, const Cand& cd) {
+    warp_visit(w, lc, x, c, [&](bool hit, const Cand& cd) {
         const bool pred = hit && cand_precedes(w, x, cd);
-        const int64_t po = pred ? off_of(w, cd.slot) : 0;
         const unsigned pb = __ballot_sync(full, pred), sb = __ballot_sync(full, hit && !pred);
         if (pred) {
             const int32_t at = np + __popc(pb & lt);
             if (at < kWarpPairs) {
-                buf[2 * at] = po;
-                buf[2 * at + 1] = po + cd.r.s;
+                buf[2 * at] = cd.slot;
+                buf[2 * at + 1] = cd.r.s;
             }
         } else if (hit) {
             const int32_t at = ns + __popc(sb & lt);
@@ -479,48 +590,66 @@ __device__ void place_short(const GridWs& w, int64_t g, int32_t policy, int64_t*
         ns += __popc(sb);
     });
     __syncwarp();
-    int64_t o;
     if (np <= kWarpPairs) {
+        for (int32_t k0 = 0; k0 < np; k0 += 32 * 4) {
+            int64_t po[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int32_t k = k0 + u * 32 + lane;
+                po[u] = k < np ? off_of(w, buf[2 * k]) : 0;
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int32_t k = k0 + u * 32 + lane;
+                if (k < np) {
+                    buf[2 * k + 1] += po[u];
+                    buf[2 * k] = po[u];
+                }
+            }
+        }
+    }
+    __syncwarp();
+    int64_t o;
+    if (np > kWarpPairs) {  // not expected (such tensors are CTA items): enumerate them again on every pass
         o = warp_fit(x.r.s, policy, [&](auto&& fn) {
-            for (int32_t k = lane; k < np; k += 32) fn(buf[2 * k], buf[2 * k + 1]);
-        });
-    } else {  // not expected (such tensors are CTA items): enumerate them again on every pass
-        o = warp_fit(x.r.s, policy, [&](auto&& fn) {
-            warp_visit(w, x, c, [&](bool hit, const Cand& cd) {
+            warp_visit(w, lc, x, c, [&](bool hit, const Cand& cd) {
                 if (hit && cand_precedes(w, x, cd)) {
                     const int64_t po = off_of(w, cd.slot);
                     fn(po, po + cd.r.s);
                 }
             });
         });
+    } else if (policy == MP_FIT_BEST && np > 32) {
+        o = warp_sorted_fit(x.r.s, policy, buf, np);
+    } else {
+        o = warp_fit(x.r.s, policy, [&](auto&& fn) {
+            for (int32_t k = lane; k < np; k += 32) fn(buf[2 * k], buf[2 * k + 1]);
+        });
     }
     if (lane == 0) st_rlx(w.off + g, o);
     __syncwarp();
     __threadfence();  // the offset before any successor's count drops
     if (lane == 0) atomicAdd(&w.ctl->placed, 1);
+    int64_t next = -1;
     if (ns <= kWarpSuccs) {
-        for (int32_t k = lane; k < ns; k += 32) {
-            const int64_t slot = sbuf[k];
-            if (atomicSub(w.cnt + slot, 1) == 1) push(w, slot);
+        for (int32_t k0 = 0; k0 < ns; k0 += 32) {
+            const int32_t k = k0 + lane;
+            const int64_t slot = k < ns ? sbuf[k] : -1;
+            const bool ready = slot >= 0 && drop(w, slot);
+            const bool warp_item = ready && !cta_item(w, slot);
+            const unsigned keep = __ballot_sync(full, warp_item && slot != w.hold);
+            const bool mine = next < 0 && keep && lane == __ffs(keep) - 1;
+            if (mine) next = slot;
+            next = __shfl_sync(full, next, keep ? __ffs(keep) - 1 : 0);
+            if (ready && !mine) push(w, slot);
         }
     } else {
-        warp_visit(w, x, c, [&](bool hit, const Cand& cd) {
-            if (hit && !cand_precedes(w, x, cd) && atomicSub(w.cnt + cd.slot, 1) == 1) push(w, cd.slot);
+        warp_visit(w, lc, x, c, [&](bool hit, const Cand& cd) {
+            if (hit && !cand_precedes(w, x, cd) && drop(w, cd.slot)) push(w, cd.slot);
         });
     }
     __syncwarp();
-}
-
-// Block max of a non-negative int64 (every thread gets it); red: 32 slots.
-__device__ __forceinline__ int64_t cta_max(int64_t v, int64_t* red) {
-    const int lane = threadIdx.x & 31, wp = threadIdx.x >> 5;
-    v = warp_max64(v);
-    if (lane == 0) red[wp] = v;
-    __syncthreads();
-    int64_t r = lane < (int)(blockDim.x >> 5) ? red[lane] : 0;
-    r = warp_max64(r);
-    __syncthreads();
-    return r;
+    return next;
 }
 
 // Exclusive prefix max (identity 0) of one value per thread; the block max in *total.
@@ -554,68 +683,134 @@ __device__ __forceinline__ int64_t cta_excl_max(int64_t v, int64_t* red, int64_t
     return r;
 }
 
-constexpr int32_t kJumpMax = 256;  // FIRST with at most this many predecessors jumps; more are sorted
+constexpr int32_t kJumpCap = 128;  // FIRST jumps at most this often before it sorts instead
+constexpr int kRegJump = 6;        // predecessor pairs per thread held in registers for the jumps
+
+// Shared state of a CTA item.
+struct LongShared {
+    int32_t np, ns, next;
+};
 
 // A tensor placed by the whole CTA (long-lived, or more predecessors than a
-// warp holds).  Its predecessors' pairs go to the shared region, then to this
-// CTA's overflow buffer (ovf).  FIRST with few of them jumps to the largest
-// conflicting end until nothing conflicts (a block reduction per jump);
-// otherwise the pairs are sorted by offset and one scan exposes every gap
-// (FIRST: the lowest that fits; BEST: the smallest that fits, the lowest on
-// ties).  Then the successors' counts drop.
-__device__ void place_long(const GridWs& w, int64_t g, int32_t policy, int64_t* region, int64_t* ovf,
-                           int64_t* red, int32_t* s_cnt) {
+// warp holds).  One pass over the candidates puts the predecessors' pairs in
+// the region (then in this CTA's overflow buffer, ovf) and lists the
+// successors after them (if too many, they are enumerated again).  FIRST jumps
+// to the largest conflicting end until nothing conflicts (pairs held in
+// registers, one block reduction per jump); if that takes more than kJumpCap
+// jumps, or for BEST, the pairs are sorted by offset and one scan exposes
+// every gap (FIRST: the lowest that fits; BEST: the smallest, the lowest on
+// ties).  Returns a successor that
+// became ready and is a CTA item, for this CTA to place next (-1 if none).
+__device__ int64_t place_long(const GridWs& w, const LongCache& lc, int64_t g, int32_t policy, int64_t* region,
+                              int64_t* ovf, int64_t* red, LongShared* sh) {
     const Node x = load_node(w, g);
-    const TraceInfo ti = w.ti[x.b];
-    const Cands c = cands_of(w, ti, x);
+    const Cands c = cands_of(w, lc.lw[x.b], lc.nl[x.b], x);
     const int32_t ncand = (c.w1 - c.w0) + c.nlong;
     const int64_t s = x.r.s;
-    if (threadIdx.x == 0) *s_cnt = 0;
+    int32_t* succ = reinterpret_cast<int32_t*>(region + 2 * kLongPredPairs);
+    if (threadIdx.x == 0) {
+        sh->np = 0;
+        sh->ns = 0;
+        sh->next = -1;
+    }
     __syncthreads();
     auto pair_at = [&](int32_t k) -> int64_t* { return k < kRegionPairs ? region + 2 * k : ovf + 2 * (k - kRegionPairs); };
     const int32_t stride = (int32_t)blockDim.x;
     for (int32_t k0 = threadIdx.x; k0 < ncand; k0 += stride * kU) {
         Cand cd[kU];
-        bool pred[kU];
+        bool hit[kU], pred[kU];
 #pragma unroll
-        for (int u = 0; u < kU; ++u) pred[u] = fetch_cand(w, x, c, k0 + u * stride, &cd[u]);
+        for (int u = 0; u < kU; ++u) hit[u] = fetch_cand(w, lc, x, c, k0 + u * stride, &cd[u]);
 #pragma unroll
-        for (int u = 0; u < kU; ++u) pred[u] = pred[u] && cand_precedes(w, x, cd[u]);
-        int64_t po[kU];
-#pragma unroll
-        for (int u = 0; u < kU; ++u) po[u] = pred[u] ? off_of(w, cd[u].slot) : 0;
+        for (int u = 0; u < kU; ++u) pred[u] = hit[u] && cand_precedes(w, x, cd[u]);
 #pragma unroll
         for (int u = 0; u < kU; ++u) {
-            if (pred[u]) {
-                int64_t* q = pair_at(atomicAdd(s_cnt, 1));
-                q[0] = po[u];
-                q[1] = po[u] + cd[u].r.s;
+            if (pred[u]) {  // (slot, size) for now; the offsets are loaded below, all at once
+                int64_t* q = pair_at(atomicAdd(&sh->np, 1));
+                q[0] = cd[u].slot;
+                q[1] = cd[u].r.s;
+            } else if (hit[u]) {
+                const int32_t at = atomicAdd(&sh->ns, 1);
+                if (at < kLongSuccs) succ[at] = (int32_t)cd[u].slot;
             }
         }
     }
     __syncthreads();
-    const int32_t P = *s_cnt;
-    int64_t o;
-    if (policy == MP_FIT_FIRST && P <= kJumpMax) {
-        o = 0;
-        for (;;) {
-            int64_t next = 0;
-            for (int32_t k = threadIdx.x; k < P; k += blockDim.x) {
-                const int64_t* q = pair_at(k);
-                const int64_t po = q[0], pe = q[1];
-                if (po < o + s && o < pe && pe > next) next = pe;
-            }
-            next = cta_max(next, red);
-            if (next <= o) break;
-            o = next;
+    const int32_t P = sh->np, S = sh->ns;
+    // the predecessors' offsets: every thread's loads in flight together; the
+    // first kRegJump * blockDim pairs also stay in registers for the jumps
+    int64_t ro[kRegJump], re[kRegJump];
+#pragma unroll
+    for (int j = 0; j < kRegJump; ++j) {
+        const int32_t k = (int32_t)threadIdx.x + j * stride;
+        ro[j] = k < P ? off_of(w, pair_at(k)[0]) : 0;
+    }
+#pragma unroll
+    for (int j = 0; j < kRegJump; ++j) {
+        const int32_t k = (int32_t)threadIdx.x + j * stride;
+        re[j] = 0;  // an empty [0, 0) pads: it never conflicts
+        if (k < P) {
+            int64_t* q = pair_at(k);
+            re[j] = ro[j] + q[1];
+            q[0] = ro[j];
+            q[1] = re[j];
         }
-    } else {
+    }
+    for (int32_t k0 = (int32_t)threadIdx.x + kRegJump * stride; k0 < P; k0 += 4 * stride) {
+        int64_t po[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int32_t k = k0 + u * stride;
+            po[u] = k < P ? off_of(w, pair_at(k)[0]) : 0;
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int32_t k = k0 + u * stride;
+            if (k < P) {
+                int64_t* q = pair_at(k);
+                q[1] += po[u];
+                q[0] = po[u];
+            }
+        }
+    }
+    __syncthreads();
+    int64_t o = 0;
+    bool sorted = policy == MP_FIT_BEST;
+    if (!sorted) {  // one barrier per jump: the warps' maxima alternate between two buffers
+        const int lane = threadIdx.x & 31, wp = threadIdx.x >> 5;
+        for (int32_t jumps = 0;; ++jumps) {
+            if (jumps == kJumpCap) {
+                sorted = true;
+                break;
+            }
+            int64_t nx = 0;
+#pragma unroll
+            for (int j = 0; j < kRegJump; ++j)
+                if (ro[j] < o + s && o < re[j] && re[j] > nx) nx = re[j];
+            for (int32_t k = (int32_t)threadIdx.x + kRegJump * stride; k < P; k += stride) {
+                const int64_t* q = pair_at(k);
+                const int64_t qo = q[0], qe = q[1];
+                if (qo < o + s && o < qe && qe > nx) nx = qe;
+            }
+            nx = warp_max64(nx);
+            int64_t* rb = red + (jumps & 1) * 32;
+            if (lane == 0) rb[wp] = nx;
+            __syncthreads();
+            int64_t m = 0;
+#pragma unroll
+            for (int k = 0; k < kGridWarps; ++k) m = max(m, rb[k]);
+            if (m <= o) break;
+            o = m;
+        }
+        __syncthreads();  // every read of the maxima done before red is used again
+    }
+    if (sorted) {
         int32_t plen = 1;
         while (plen < P) plen <<= 1;
-        // sort by offset: in the shared region if it holds plen pairs, else all
-        // of them in the overflow buffer (it holds a power of two at least
-        // max_tensors): ovf[0, P - r) already holds the pairs past the
-        // region's r = min(P, R), and the region's go behind them
+        // sort by offset: in the region's pair part if it holds plen pairs, else
+        // all of them in the overflow buffer (a power of two at least
+        // max_tensors): ovf[0, P - r) already holds the pairs past the region's
+        // r = min(P, kRegionPairs), and the region's go behind them
         int64_t* arr = region;
         if (plen > kRegionPairs) {
             const int32_t r = min(P, kRegionPairs);
@@ -673,67 +868,145 @@ __device__ void place_long(const GridWs& w, int64_t g, int32_t policy, int64_t* 
     __syncthreads();
     __threadfence();
     if (threadIdx.x == 0) atomicAdd(&w.ctl->placed, 1);
-    for (int32_t k0 = threadIdx.x; k0 < ncand; k0 += stride * kU) {
-        Cand cd[kU];
-        bool succ[kU];
+    auto ready = [&](int64_t slot) {
+        if (!drop(w, slot)) return;
+        if (slot != w.hold && cta_item(w, slot) && atomicCAS(&sh->next, -1, (int32_t)slot) == -1) return;
+        push(w, slot);
+    };
+    if (S <= kLongSuccs) {  // the drops of a thread's successors in flight together
+        for (int32_t k0 = threadIdx.x; k0 < S; k0 += 4 * stride) {
+            int32_t old4[4];
+            int64_t sl[4];
 #pragma unroll
-        for (int u = 0; u < kU; ++u) succ[u] = fetch_cand(w, x, c, k0 + u * stride, &cd[u]);
+            for (int u = 0; u < 4; ++u) {
+                const int32_t k = k0 + u * stride;
+                sl[u] = k < S ? succ[k] : -1;
+                old4[u] = sl[u] >= 0 ? atomicSub(w.cnt + sl[u], 1) : 0;
+            }
 #pragma unroll
-        for (int u = 0; u < kU; ++u) succ[u] = succ[u] && !cand_precedes(w, x, cd[u]);
-        int32_t old[kU];
+            for (int u = 0; u < 4; ++u) {
+                if (old4[u] != 1) continue;
+                const int64_t slot = sl[u];
+                if (slot != w.hold && cta_item(w, slot) && atomicCAS(&sh->next, -1, (int32_t)slot) == -1) continue;
+                push(w, slot);
+            }
+        }
+    } else {
+        for (int32_t k0 = threadIdx.x; k0 < ncand; k0 += stride * kU) {
+            Cand cd[kU];
+            bool sc[kU];
 #pragma unroll
-        for (int u = 0; u < kU; ++u) old[u] = succ[u] ? atomicSub(w.cnt + cd[u].slot, 1) : 0;
+            for (int u = 0; u < kU; ++u) sc[u] = fetch_cand(w, lc, x, c, k0 + u * stride, &cd[u]);
 #pragma unroll
-        for (int u = 0; u < kU; ++u)
-            if (succ[u] && old[u] == 1) push(w, cd[u].slot);
+            for (int u = 0; u < kU; ++u)
+                if (sc[u] && !cand_precedes(w, x, cd[u])) ready(cd[u].slot);
+        }
     }
     __syncthreads();
+    const int64_t next = sh->next;
+    __syncthreads();
+    return next;
 }
 
-// Waits (bounded) until a queue slot is filled and returns its entry, or
-// returns -1 once every tensor is placed, another CTA gave up, or nothing was
-// queued or placed anywhere for kGridSpinCycles (then it raises the flag).
-__device__ int32_t take_slot(const GridWs& w, const int32_t* slot, int32_t total) {
+// Waits (bounded) until queue slot h (of the queue whose fill count is *tail)
+// is filled and returns its entry, or returns -1 once every tensor is placed,
+// another worker gave up, or nothing was queued or placed anywhere for
+// kGridSpinCycles (then it raises the flag).  Only the slot is polled often,
+// at a rate set by its distance from the queue's fill point; the shared
+// counters are read every eighth poll, so idle workers load the L2 little.
+__device__ int32_t take_slot(const GridWs& w, const int32_t* queue, const int32_t* tail, int32_t h,
+                             int32_t total) {
     GridCtl* ctl = w.ctl;
-    long long idle_since = 0;
-    int32_t seen = -1;
+    long long idle_since = clock64();
+    int32_t seen = -1, dist = 0;
     for (int32_t polls = 0;; ++polls) {
-        const int32_t v = ld_rlx(slot);
+        const int32_t v = ld_rlx(queue + h);
         if (v >= 0) return v;
-        if (polls < 4) continue;  // an entry due at any moment: poll it first
-        if (ld_rlx(&ctl->fail)) return -1;
-        const int32_t placed = ld_rlx(&ctl->placed);
-        if (placed >= total) return -1;
-        const int32_t act = placed + ld_rlx(&ctl->tail_s) + ld_rlx(&ctl->tail_l);
-        if (act != seen) {
-            seen = act;
-            idle_since = clock64();
-        } else if (clock64() - idle_since > kGridSpinCycles) {
-            atomicExch(&ctl->fail, 1);
-            return -1;
+        if ((polls & 7) == 0) {
+            if (ld_rlx(&ctl->fail)) return -1;
+            const int32_t placed = ld_rlx(&ctl->placed);
+            if (placed >= total) return -1;
+            const int32_t t = ld_rlx(tail);
+            dist = h - t;
+            const int32_t act = placed + ld_rlx(&ctl->tail_s) + ld_rlx(&ctl->tail_l);
+            if (act != seen) {
+                seen = act;
+                idle_since = clock64();
+            } else if (clock64() - idle_since > kGridSpinCycles) {
+                atomicExch(&ctl->fail, 1);
+                return -1;
+            }
         }
-        __nanosleep(polls < 64 ? 32 : 256);
+        __nanosleep(dist <= 0 ? 32 : dist <= 4 ? 128 : dist <= 64 ? 512 : 2048);
     }
 }
 
-// The persistent grid: all warps first count predecessors; then the first
-// long_ctas CTAs place CTA items (thread 0 takes the next long-queue slot for
-// the whole CTA) and every warp of the others places warp items (each takes
-// the next short-queue slot for itself).  A worker waits only for the entry
-// of the slot it took; it never holds one entry while waiting for another, and
-// the lowest-ranked unplaced tensor of a trace is always queued, so a taken
-// slot is always filled in the end.  With w.hold >= 0 (tests only) the tensor
-// of that slot is never queued, so the flow starves and the wait runs out.
+// The persistent grid.  Each CTA first copies the batch's long-lived records
+// into its shared-memory cache (if they fit), then all warps count
+// predecessors; then the first long_ctas CTAs place CTA items (thread 0 takes
+// the next long-queue slot for the whole CTA) and every warp of the others
+// places warp items (each takes the next short-queue slot for itself).  A
+// worker that makes a successor of its own kind ready places it next instead
+// of queueing it.  A worker waits only for the entry of the slot it took and
+// never holds one entry while waiting for another; the lowest-ranked unplaced
+// tensor of a trace is always queued or being placed, so a taken slot is
+// always filled in the end.  With w.hold >= 0 (tests only) the tensor of that
+// slot is never queued, so the flow starves and the wait runs out.
 __global__ void __launch_bounds__(kGridThreads, 1)
 k_grid_flow(mp_batch bt, int32_t policy, GridWs w, int32_t long_ctas) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     __shared__ int64_t red[72];
-    __shared__ int32_t s_long, s_cnt;
+    __shared__ int32_t s_long, s_cbase[kGridMaxTraces + 1], s_lw[kGridMaxTraces], s_nl[kGridMaxTraces];
+    __shared__ LongShared s_sh;
     int64_t* region = reinterpret_cast<int64_t*>(smem_raw);
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int64_t M = w.M;
     const int64_t slots = (int64_t)bt.n_traces * M;
     GridCtl* ctl = w.ctl;
+
+    // the long-lived cache: trace b's records at [s_cbase[b], s_cbase[b + 1])
+    LongCache lc;
+    {
+        unsigned char* cache = smem_raw + kRegionBytes;
+        lc.s = reinterpret_cast<int64_t*>(cache);
+        lc.a = reinterpret_cast<int32_t*>(cache + (size_t)kLongCache * 8);
+        lc.f = lc.a + kLongCache;
+        lc.q = lc.f + kLongCache;
+        lc.base = nullptr;
+        lc.lw = s_lw;
+        lc.nl = s_nl;
+        if (threadIdx.x < bt.n_traces) {
+            const TraceInfo* tb = w.ti + threadIdx.x;
+            s_lw[threadIdx.x] = tb->ok ? tb->lw : 1;
+            s_nl[threadIdx.x] = tb->ok ? tb->nlong : 0;
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            int32_t at = 0;
+            for (int32_t b = 0; b < bt.n_traces; ++b) {
+                s_cbase[b] = at;
+                at += s_nl[b];
+            }
+            s_cbase[bt.n_traces] = at;
+        }
+        __syncthreads();
+        if (s_cbase[bt.n_traces] <= kLongCache) {
+            for (int32_t b = 0; b < bt.n_traces; ++b) {
+                const int32_t nl = s_cbase[b + 1] - s_cbase[b];
+                for (int32_t k = threadIdx.x; k < nl; k += blockDim.x) {
+                    const int32_t q = __ldg(w.ll + (int64_t)b * M + k);
+                    const GRec r = load_rec(w, (int64_t)b * M + q);
+                    const int32_t i = s_cbase[b] + k;
+                    lc.s[i] = r.s;
+                    lc.a[i] = r.a;
+                    lc.f[i] = r.f;
+                    lc.q[i] = q;
+                }
+            }
+            lc.base = s_cbase;
+        }
+        __syncthreads();
+    }
 
     // counts: a warp per tensor; the class is set before the count is added
     {
@@ -742,11 +1015,10 @@ k_grid_flow(mp_batch bt, int32_t policy, GridWs w, int32_t long_ctas) {
             const int32_t b = (int32_t)(g / M), p = (int32_t)(g - (int64_t)b * M);
             const TraceInfo* tip = w.ti + b;
             if (!tip->ok || p >= tip->n) continue;
-            const TraceInfo ti = *tip;
             const Node x = load_node(w, g);
-            const Cands c = cands_of(w, ti, x);
+            const Cands c = cands_of(w, lc.lw[b], lc.nl[b], x);
             int32_t np = 0;
-            warp_visit(w, x, c, [&](bool hit, const Cand& cd) {
+            warp_visit(w, lc, x, c, [&](bool hit, const Cand& cd) {
                 np += __popc(__ballot_sync(0xffffffffu, hit && cand_precedes(w, x, cd)));
             });
             if (lane == 0) {
@@ -760,31 +1032,38 @@ k_grid_flow(mp_batch bt, int32_t policy, GridWs w, int32_t long_ctas) {
     const int32_t total = ctl->total;
     if ((int32_t)blockIdx.x < long_ctas) {
         int64_t* ovf = w.ovf_pairs > 0 ? w.ovf + (int64_t)blockIdx.x * 2 * w.ovf_pairs : nullptr;
+        int64_t next = -1;
         for (;;) {
-            if (threadIdx.x == 0) {
-                const int32_t h = atomicAdd(&ctl->head_l, 1);
-                s_long = h < total ? take_slot(w, w.ql + h, total) : -1;
-                __threadfence();  // the predecessors' offsets after the entry
+            if (next < 0) {
+                if (threadIdx.x == 0) {
+                    const int32_t h = atomicAdd(&ctl->head_l, 1);
+                    s_long = h < total ? take_slot(w, w.ql, &ctl->tail_l, h, total) : -1;
+                    __threadfence();  // the predecessors' offsets after the entry
+                }
+                __syncthreads();
+                next = s_long;
+                __syncthreads();
+                if (next < 0) break;
             }
-            __syncthreads();
-            const int32_t v = s_long;
-            if (v < 0) break;
             __threadfence();
-            place_long(w, v, policy, region, ovf, red, &s_cnt);
+            next = place_long(w, lc, next, policy, region, ovf, red, &s_sh);
         }
     } else {
-        int64_t* buf = region + (int64_t)warp * 2 * (kRegionPairs / kGridWarps);
+        int64_t* buf = region + (int64_t)warp * (kWarpBytes / 8);
+        int64_t next = -1;
         for (;;) {
-            int32_t v = -1;
-            if (lane == 0) {
-                const int32_t h = atomicAdd(&ctl->head_s, 1);
-                v = h < total ? take_slot(w, w.qs + h, total) : -1;
-                __threadfence();
+            if (next < 0) {
+                int32_t v = -1;
+                if (lane == 0) {
+                    const int32_t h = atomicAdd(&ctl->head_s, 1);
+                    v = h < total ? take_slot(w, w.qs, &ctl->tail_s, h, total) : -1;
+                    __threadfence();
+                }
+                next = __shfl_sync(0xffffffffu, v, 0);
+                if (next < 0) break;
             }
-            v = __shfl_sync(0xffffffffu, v, 0);
-            if (v < 0) break;
             __threadfence();
-            place_short(w, v, policy, buf);
+            next = place_short(w, lc, next, policy, buf);
         }
     }
 }

@@ -28,7 +28,8 @@ constexpr size_t kProfileSmemLimit = kSmemCeiling;
 constexpr size_t kValidateSmemLimit = kSmemCeiling;
 constexpr size_t kPlanSmemLimit = kSmemCeiling;
 
-// Raises the kernel's dynamic shared memory ceiling once per device.
+// Raises the kernel's dynamic shared memory ceiling once per device (to
+// kSmemCeiling, or to `bytes` for a kernel that asks for more).
 cudaError_t set_smem_limit(const void* func, size_t bytes);
 
 // CTAs of `func` (threads, dynamic shared memory smem) the current device holds

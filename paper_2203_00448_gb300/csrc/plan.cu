@@ -991,92 +991,80 @@ __device__ __forceinline__ W block_excl_scan_w(W v, int64_t* red, W* total) {
     return block_excl_scan<W>(v, reinterpret_cast<W*>(red), total);
 }
 
-// Places a component none of whose members lives longer than kLongLife
-// steps with one warp, in priority order 32 ranks at a time; ord: its members'
-// positions by rank.  Every member of a batch depends only on lower ranks:
-// those of earlier batches are final, and inside the batch the offsets are
-// found by rounds in which every lane recomputes its member's offset from the
-// current offsets of its predecessors (one snapshot per round).  The
-// dependencies are acyclic, so the system has one fixed point -- the
-// sequential definition's offsets -- and a round that changes nothing has
-// reached it; a member whose longest chain of predecessors inside the batch
-// has d links is final after round d, so at most 33 rounds are needed.  The
-// predecessors of a member are among the members of its window (allocated in
-// (a - lw, f)); up to 64 positions they are kept as a bit mask, else tested on
-// every pass.  Returns this lane's largest end; sets *fail to 2 if a batch does
-// not settle (an inconsistency, never expected).
+// A window of more than this many alloc-order positions has no predecessor
+// mask; the walk then tests its candidates on every pass.
+constexpr int32_t kMaskBits = 64;
+constexpr int32_t kUnmasked = 1 << 30;  // flag in the window start word
+
+// Walks a component none of whose members lives longer than kLongLife steps,
+// one thread, in priority order: ord[r] is the member of rank r, W0[x] the
+// first position of member x's window (with kUnmasked when it has no mask) and
+// PM[x] the mask of its predecessors in the window, both computed beforehand
+// by the whole CTA.  Every predecessor of a member was placed earlier in the
+// same walk, so the gap search sees final offsets: this is the sequential
+// definition itself, at the cost of one short loop per member.  Returns the
+// largest end.
 template <typename I, typename W>
-__device__ W place_comp_rounds(const ARec<I, W>* AR, W* OFFP, const int32_t* BEND, const int32_t* ord, int32_t p0,
-                               int32_t c, int32_t lw, int32_t policy, volatile int32_t* fail) {
-    const unsigned full = 0xffffffffu;
-    const int lane = threadIdx.x & 31;
-    volatile W* voff = OFFP;
+__device__ W walk_comp(const ARec<I, W>* AR, W* OFFP, const int32_t* BEND, const int32_t* ord, const int32_t* W0,
+                       const uint64_t* PM, int32_t p0, int32_t c, int32_t policy) {
     W mx = 0;
-    for (int32_t r0 = 0; r0 < c; r0 += 32) {
-        const int32_t r = r0 + lane;
-        const bool act = r < c;
-        int32_t x = -1, w0 = 0, w1 = 0;
-        ARec<I, W> me{};
-        uint64_t pm = 0;
-        if (act) {
-            x = ord[r];
-            me = AR[x];
-            w0 = max(p0, (int32_t)me.a >= lw ? BEND[(int32_t)me.a - lw] : 0);
-            w1 = min(p0 + c, BEND[(int32_t)me.f - 1]);
-            if (w1 - w0 <= 64) {
-                for (int32_t q = w0; q < w1; ++q) {
-                    if (q == x) continue;
-                    const ARec<I, W> o = AR[q];
-                    if ((int32_t)o.a < (int32_t)me.f && (int32_t)me.a < (int32_t)o.f && precedes(o, me))
-                        pm |= 1ull << (q - w0);
+    for (int32_t r = 0; r < c; ++r) {
+        const int32_t x = ord[r];
+        const ARec<I, W> me = AR[x];
+        const int32_t wv = W0[x];
+        const int32_t w0 = wv & (kUnmasked - 1);
+        const uint64_t pm = PM[x];
+        // up to kRegPreds predecessors are loaded into registers once, and the
+        // passes of the gap search then read no memory
+        constexpr int kRegPreds = 8;
+        const bool in_regs = !(wv & kUnmasked) && __popcll(pm) <= kRegPreds;
+        W ro[kRegPreds], re[kRegPreds];
+        if (in_regs) {
+            uint64_t m = pm;
+#pragma unroll
+            for (int j = 0; j < kRegPreds; ++j) {
+                ro[j] = 0;
+                re[j] = 0;  // an empty interval [0, 0) never conflicts and never raises the top
+                if (m) {
+                    const int32_t q = w0 + __ffsll((long long)m) - 1;
+                    m &= m - 1;
+                    ro[j] = OFFP[q];
+                    re[j] = (W)(ro[j] + AR[q].s);
                 }
             }
-            voff[x] = 0;
         }
-        const bool masked = w1 - w0 <= 64;
         auto each = [&](auto&& fn) {
-            if (masked) {
+            if (in_regs) {
+#pragma unroll
+                for (int j = 0; j < kRegPreds; ++j) fn(ro[j], re[j]);
+            } else if (!(wv & kUnmasked)) {
                 for (uint64_t m = pm; m; m &= m - 1) {
                     const int32_t q = w0 + __ffsll((long long)m) - 1;
-                    const W o = voff[q];
+                    const W o = OFFP[q];
                     fn(o, (W)(o + AR[q].s));
                 }
             } else {
+                const int32_t w1 = min(p0 + c, BEND[(int32_t)me.f - 1]);
                 for (int32_t q = w0; q < w1; ++q) {
                     if (q == x) continue;
                     const ARec<I, W> oq = AR[q];
                     if ((int32_t)oq.a < (int32_t)me.f && (int32_t)me.a < (int32_t)oq.f && precedes(oq, me)) {
-                        const W o = voff[q];
+                        const W o = OFFP[q];
                         fn(o, (W)(o + oq.s));
                     }
                 }
             }
         };
-        __syncwarp();
-        W o = 0;
-        for (int round = 0;; ++round) {
-            W on = 0;
-            if (act) {
-                if (policy == MP_FIT_FIRST) {
-                    on = fit_first_scan<W>(me.s, each);
-                } else {
-                    W top = 0;
-                    each([&](W, W pe) { top = pe > top ? pe : top; });
-                    on = fit_best_scan<W>(me.s, top, each);
-                }
-            }
-            const bool changed = act && on != o;
-            __syncwarp();
-            if (act) voff[x] = on;
-            o = on;
-            __syncwarp();
-            if (!__any_sync(full, changed)) break;
-            if (round >= 40) {
-                *fail = 2;
-                break;
-            }
+        W o;
+        if (policy == MP_FIT_FIRST) {
+            o = fit_first_scan<W>(me.s, each);
+        } else {
+            W top = 0;
+            each([&](W, W pe) { top = pe > top ? pe : top; });
+            o = fit_best_scan<W>(me.s, top, each);
         }
-        if (act) mx = o + me.s > mx ? o + me.s : mx;
+        OFFP[x] = o;
+        mx = o + me.s > mx ? o + me.s : mx;
     }
     return mx;
 }
@@ -1085,8 +1073,8 @@ __device__ W place_comp_rounds(const ARec<I, W>* AR, W* OFFP, const int32_t* BEN
 // defers traces with components above kDeferComp, and with its data in the
 // workspace, every trace that needs this tier).  Each is first sorted into
 // priority order by the whole CTA.  Components whose members all live at most
-// kLongLife steps are then placed concurrently, a warp each, by rounds
-// (place_comp_rounds).  In the others the long-lived members cut the priority
+// kLongLife steps are then placed concurrently, one thread walking each
+// (walk_comp).  In the others the long-lived members cut the priority
 // order into runs of short-lived ones, which the warps place together from a
 // ready queue, each long-lived one then by the whole CTA.  Returns this
 // thread's largest end.
@@ -1118,20 +1106,54 @@ __device__ __forceinline__ W large_tier(const ARec<I, W>* AR, W* OFFP, const int
         for (int32_t r = threadIdx.x; r < sz; r += blockDim.x) ORD[p0 + r] = sortbuf[r];
     }
     __syncthreads();
-    // 2. components without long-lived members: a warp each, all at once
-    for (int32_t qc = warp; qc < nx; qc += nwarps) {
+    // 2. components without long-lived members.  First the whole CTA gives
+    // every member its window and the mask of its predecessors there (W0
+    // aliases HR, PM the CNT and QUE words, both free until step 3; W0[p0] = -1
+    // marks a component left to step 3); then one thread walks each component,
+    // all components at once.
+    int32_t* W0 = HR;
+    uint64_t* PM = reinterpret_cast<uint64_t*>(CNT);
+    for (int32_t qc = 0; qc < nx; ++qc) {
         const int32_t p0 = LST[qc], sz = comp_size(SB, NW, p0, n);
-        bool any_long = false;
-        uint32_t lw = 1;
-        for (int32_t k = (threadIdx.x & 31); k < sz; k += 32) {
+        int32_t any_long = 0, lw = 1;
+        for (int32_t k = threadIdx.x; k < sz; k += blockDim.x) {
             const int32_t life = (int32_t)AR[p0 + k].f - (int32_t)AR[p0 + k].a;
-            any_long |= life > kLongLife;
-            if (life <= kLongLife) lw = max(lw, (uint32_t)life);
+            any_long |= life > kLongLife ? 1 : 0;
+            if (life <= kLongLife) lw = max(lw, life);
         }
-        if (__any_sync(0xffffffffu, any_long)) continue;  // step 3
-        const W e = place_comp_rounds<I, W>(AR, OFFP, BEND, ORD + p0, p0, sz,
-                                            (int32_t)__reduce_max_sync(0xffffffffu, lw), policy, s_fail);
-        mx = max(mx, e);
+        if (__syncthreads_or(any_long)) {
+            if (threadIdx.x == 0) W0[p0] = -1;
+            continue;
+        }
+        int64_t lw_max;
+        block_excl_max((int64_t)lw, red, &lw_max);
+        const int32_t lwc = (int32_t)lw_max;
+        for (int32_t x = p0 + threadIdx.x; x < p0 + sz; x += blockDim.x) {
+            const ARec<I, W> me = AR[x];
+            const int32_t w0 = max(p0, (int32_t)me.a >= lwc ? BEND[(int32_t)me.a - lwc] : 0);
+            const int32_t w1 = min(p0 + sz, BEND[(int32_t)me.f - 1]);
+            uint64_t pm = 0;
+            if (w1 - w0 <= kMaskBits) {
+                for (int32_t q = w0; q < w1; ++q) {
+                    if (q == x) continue;
+                    const ARec<I, W> o = AR[q];
+                    if ((int32_t)o.a < (int32_t)me.f && (int32_t)me.a < (int32_t)o.f && precedes(o, me))
+                        pm |= 1ull << (q - w0);
+                }
+            }
+            W0[x] = w0 | (w1 - w0 <= kMaskBits ? 0 : kUnmasked);
+            PM[x] = pm;
+        }
+    }
+    __syncthreads();
+    {
+        const int lane = threadIdx.x & 31;
+        for (int32_t qc = warp + nwarps * lane; qc < nx; qc += blockDim.x) {
+            const int32_t p0 = LST[qc];
+            if (W0[p0] < 0) continue;
+            const W e = walk_comp<I, W>(AR, OFFP, BEND, ORD + p0, W0, PM, p0, comp_size(SB, NW, p0, n), policy);
+            mx = max(mx, e);
+        }
     }
     __syncthreads();
     // 3. components with long-lived members, one after the other: their
@@ -1621,7 +1643,7 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
                 out.conflict[2 * b + 1] = good ? -1 : (int32_t)(key & 0xffffffffu);
             }
         }
-        status[b] = s_fail == 2 ? MP_EINTERNAL : s_fail ? MP_ETIMEOUT : MP_OK;
+        status[b] = s_fail ? MP_ETIMEOUT : MP_OK;
     }
 }
 
