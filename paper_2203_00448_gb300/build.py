@@ -77,6 +77,41 @@ def build(force: bool = False, verbose: bool = False, extra_flags=None) -> str:
     return LIB_PATH
 
 
+TEST_HOOKS_DIR = os.path.join(BUILD_DIR, "test_hooks")
+TEST_HOOKS_LIB = os.path.join(TEST_HOOKS_DIR, "libmemplan_test_hooks.so")
+# Test builds: the entry point mp_test_plan_hold, and bounds on the planner's
+# waits of about 8 ms instead of about a second.
+TEST_HOOKS_FLAGS = ["-DMP_TEST_HOOKS", "-DMP_TEST_SPIN_CYCLES=(1ll<<24)", "-DMP_TEST_GRID_SPIN_CYCLES=(1ll<<24)"]
+
+
+def build_test_hooks(force: bool = False) -> str:
+    """Compiles the library a second time with the test hooks into _build/
+    (never loaded by the package itself); returns its path."""
+    if not force and os.path.exists(TEST_HOOKS_LIB) and all(
+            os.path.getmtime(p) <= os.path.getmtime(TEST_HOOKS_LIB) for p in _inputs()):
+        return TEST_HOOKS_LIB
+    os.makedirs(TEST_HOOKS_DIR, exist_ok=True)
+    cc = nvcc()
+    flags = NVCC_FLAGS + TEST_HOOKS_FLAGS
+
+    def compile_one(src):
+        obj = os.path.join(TEST_HOOKS_DIR, os.path.basename(src)[:-3] + ".o")
+        r = subprocess.run([cc, *ARCH, *flags, "-c", src, "-o", obj], capture_output=True, text=True)
+        if r.returncode != 0:
+            raise RuntimeError(f"nvcc failed on {src}:\n{r.stdout}\n{r.stderr}")
+        return obj
+
+    srcs = sources()
+    with ThreadPoolExecutor(max_workers=min(len(srcs), os.cpu_count() or 4)) as ex:
+        objs = list(ex.map(compile_one, srcs))
+    tmp = TEST_HOOKS_LIB + f".tmp{os.getpid()}"
+    r = subprocess.run([cc, *ARCH, "-shared", "-o", tmp, *objs, "-lcudart"], capture_output=True, text=True)
+    if r.returncode != 0:
+        raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
+    os.replace(tmp, TEST_HOOKS_LIB)
+    return TEST_HOOKS_LIB
+
+
 if __name__ == "__main__":
     import sys
 

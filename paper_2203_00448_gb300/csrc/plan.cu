@@ -70,7 +70,11 @@ constexpr int kCached = 4;           // tensors per thread kept in registers bet
 constexpr int32_t kLongLife = 32;    // CTA tier: members living longer than this many steps are listed apart
 constexpr int32_t kPredBuf = 512;    // CTA tier, data in the workspace: predecessors gathered per warp
 constexpr int32_t kLongStage = 2048; // CTA tier, data in the workspace: long-lived members staged in shared memory
+#ifdef MP_TEST_SPIN_CYCLES
+constexpr long long kSpinCycles = MP_TEST_SPIN_CYCLES;  // test builds: a short bound
+#else
 constexpr long long kSpinCycles = 1ll << 31;  // a wait for another warp longer than this is a fault
+#endif
 constexpr int32_t kValWide = 64;     // validation: windows longer than this get a warp each
 constexpr int32_t kFlowWarps = 16;   // warps that take members from a run's ready queue
 constexpr int32_t kDeferComp = 1024;  // the 32-bit launch (data in shared memory) defers larger components
@@ -457,6 +461,7 @@ struct Comp {
     const int32_t* ord;
     const int32_t* hr;
     int32_t p0, c, nl, lw;
+    int32_t hold;  // test builds: a member never queued (-1: none)
     LongStage<W> st;
     bool staged;
 
@@ -541,6 +546,7 @@ __device__ W place_run(const Comp<I, W>& cp, int32_t r0, int32_t r1, int32_t nl_
         return (int32_t)o.a < (int32_t)me.f && (int32_t)me.a < (int32_t)o.f;
     };
     auto push = [&](int32_t x) {
+        if (x == cp.hold) return;  // only in test builds: the run then starves and its waits run out
         const int32_t at = atomicAdd(tail, 1);
         vque[at] = x;
     };
@@ -1082,7 +1088,7 @@ template <typename I, typename W, bool kSmem>
 __device__ __forceinline__ W large_tier(const ARec<I, W>* AR, W* OFFP, const int32_t* BEND, const uint32_t* SB,
                                      const int32_t* NW, const int32_t* LST, int32_t nx, int32_t n, int32_t* ORD, int32_t* HR, int32_t* CNT, int32_t* QUE, int64_t* bo, int64_t* be,
                                      unsigned char* smem_raw, int32_t policy, int64_t* red, int32_t* s_cnt,
-                                     int32_t* s_tail, int32_t* s_fail) {
+                                     int32_t* s_tail, int32_t* s_fail, int32_t hold) {
     const int warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
     W mx = 0;
     W* scratch = nullptr;
@@ -1204,6 +1210,7 @@ __device__ __forceinline__ W large_tier(const ARec<I, W>* AR, W* OFFP, const int
         cp.lw = (int32_t)lw_max;
         cp.st = st;
         cp.staged = !kSmem && nl <= kLongStage;
+        cp.hold = hold;
         for (int32_t k = 0; k <= nl; ++k) {
             const int32_t r0 = k == 0 ? 0 : HR[k - 1] + 1, r1 = k < nl ? HR[k] : sz;
             if (r1 > r0) {  // the short-lived run between two long-lived members
@@ -1228,6 +1235,16 @@ __device__ __forceinline__ W large_tier(const ARec<I, W>* AR, W* OFFP, const int
 
     return mx;
 }
+
+// Test builds (MP_TEST_HOOKS) can name one member, by trace and alloc-order
+// position, that the CTA tier never queues, so that a run starves and its
+// bounded waits run out; in every other build no member is held.
+#ifdef MP_TEST_HOOKS
+__device__ int32_t g_test_hold[2] = {-1, -1};
+__device__ __forceinline__ int32_t test_hold_position(int b) { return b == g_test_hold[0] ? g_test_hold[1] : -1; }
+#else
+__device__ __forceinline__ int32_t test_hold_position(int) { return -1; }
+#endif
 
 // ------------------------------------------------------------- the kernel
 
@@ -1576,7 +1593,8 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
     if (s_base[kBins] > s_base[kBinCta]) {
         const W e = large_tier<I, W, kSmem>(AR, OFFP, BEND, SB, NW, LST + s_base[kBinCta], s_base[kBins] - s_base[kBinCta],
                                             n, ORD, HR, CNT,
-                                            QUE, bo, be, smem_raw, policy, red, &s_cnt, &s_tail, &s_fail);
+                                            QUE, bo, be, smem_raw, policy, red, &s_cnt, &s_tail, &s_fail,
+                                            test_hold_position(b));
         mx = max(mx, e);
     }
 
@@ -1809,3 +1827,33 @@ cudaError_t launch_plan_fused(const mp_batch& bt, int32_t policy, int64_t* profi
 }
 
 }  // namespace mp
+
+#ifdef MP_TEST_HOOKS
+// Test builds only: greedy_by_size as mp_plan_greedy_by_size, except that the
+// member at alloc-order position hold_pos of trace hold_trace is never queued
+// (the grid-wide planner for batches of a few large traces, the CTA tier's
+// ready queue otherwise), so the planner's bounded waits run out and that
+// trace reports MP_ETIMEOUT while the others are planned as usual.
+extern "C" __attribute__((visibility("default"))) mp_status mp_test_plan_hold(
+    const mp_batch* batch, mp_fit_policy policy, int64_t* offsets, int64_t* plan_peak, int32_t* trace_status,
+    void* workspace, size_t workspace_bytes, int32_t hold_trace, int32_t hold_pos, void* stream) {
+    static const int32_t none[2] = {-1, -1};
+    static int32_t held[2];
+    if (batch == nullptr || workspace_bytes < mp::plan_workspace_bytes(*batch)) return MP_EINVAL;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (mp::grid_path(*batch)) {
+        const int64_t slot = (int64_t)hold_trace * batch->max_tensors + hold_pos;
+        return mp::launch_grid_plan(*batch, policy, offsets, plan_peak, trace_status, workspace, (int32_t)slot, st) ==
+                       cudaSuccess
+                   ? MP_OK
+                   : MP_ECUDA;
+    }
+    held[0] = hold_trace;
+    held[1] = hold_pos;
+    cudaError_t e = cudaMemcpyToSymbol(mp::g_test_hold, held, sizeof(held));
+    if (e == cudaSuccess) e = mp::launch_plan(*batch, policy, offsets, plan_peak, trace_status, workspace, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    const cudaError_t e2 = cudaMemcpyToSymbol(mp::g_test_hold, none, sizeof(none));
+    return e == cudaSuccess && e2 == cudaSuccess ? MP_OK : MP_ECUDA;
+}
+#endif
