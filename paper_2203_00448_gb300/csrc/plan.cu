@@ -292,6 +292,41 @@ __device__ __forceinline__ int64_t warp_min_w(int64_t v) {
     return (int64_t)(((uint64_t)hi << 32) | lo);
 }
 
+// BEST by one warp over the predecessor pairs each lane supplies through
+// each(fn): the free holes below the top walked in address order, the
+// smallest that fits kept, the lowest on ties, else the top.
+template <typename W, typename Each>
+__device__ W warp_best_fit(W s, Each&& each) {
+    W top = 0;
+    each([&](W, W pe) { top = pe > top ? pe : top; });
+    top = warp_max_w(top);
+    W c = 0, best_len = w_none<W>(), best = top;
+    while (c < top) {
+        for (;;) {  // move c off any predecessor that covers it
+            W cov = 0;
+            each([&](W po, W pe) {
+                if (po <= c && c < pe && pe > cov) cov = pe;
+            });
+            cov = warp_max_w(cov);
+            if (cov <= c) break;
+            c = cov;
+        }
+        if (c >= top) break;
+        W ns = w_none<W>();
+        each([&](W po, W) {
+            if (po > c && po < ns) ns = po;
+        });
+        ns = warp_min_w(ns);
+        const W len = ns - c;
+        if (len >= s && len < best_len) {
+            best_len = len;
+            best = c;
+        }
+        c = ns;
+    }
+    return best;
+}
+
 // Places the component at positions [p0, p0 + c), c <= 32, with one warp (a
 // tensor per lane); every lane must call it.  Writes OFFP; returns the
 // largest end.
@@ -997,79 +1032,111 @@ __device__ __forceinline__ W block_excl_scan_w(W v, int64_t* red, W* total) {
     return block_excl_scan<W>(v, reinterpret_cast<W*>(red), total);
 }
 
+// Components of more than kWalkMin members without long-lived ones are walked
+// by one warp (walk_comp): cheapest when the dependencies form long chains,
+// as in a network whose activations are all alike.  Smaller ones go to the
+// ready-queue runs, whose warps overlap the independent members of a shallow
+// dependency graph.
+constexpr int32_t kWalkMin = 64;
+
 // A window of more than this many alloc-order positions has no predecessor
 // mask; the walk then tests its candidates on every pass.
 constexpr int32_t kMaskBits = 64;
 constexpr int32_t kUnmasked = 1 << 30;  // flag in the window start word
 
-// Walks a component none of whose members lives longer than kLongLife steps,
-// one thread, in priority order: ord[r] is the member of rank r, W0[x] the
+// Walks a component none of whose members lives longer than kLongLife steps
+// with one warp, in priority order: ord[r] is the member of rank r, W0[x] the
 // first position of member x's window (with kUnmasked when it has no mask) and
 // PM[x] the mask of its predecessors in the window, both computed beforehand
 // by the whole CTA.  Every predecessor of a member was placed earlier in the
 // same walk, so the gap search sees final offsets: this is the sequential
-// definition itself, at the cost of one short loop per member.  Returns the
+// definition itself.  Lane l holds the predecessors at window positions l and
+// l + 32, so a member costs one parallel load and a few warp reductions.  The
+// next member's entries are loaded while the current one is placed (they do
+// not depend on any offset).  Every lane must call it; returns this lane's
 // largest end.
 template <typename I, typename W>
 __device__ W walk_comp(const ARec<I, W>* AR, W* OFFP, const int32_t* BEND, const int32_t* ord, const int32_t* W0,
                        const uint64_t* PM, int32_t p0, int32_t c, int32_t policy) {
+    const int lane = threadIdx.x & 31;
+    volatile W* voff = OFFP;
     W mx = 0;
+    int32_t xn = c > 0 ? ord[0] : 0;
+    ARec<I, W> men = AR[xn];
+    int32_t wvn = W0[xn];
+    uint64_t pmn = PM[xn];
     for (int32_t r = 0; r < c; ++r) {
-        const int32_t x = ord[r];
-        const ARec<I, W> me = AR[x];
-        const int32_t wv = W0[x];
-        const int32_t w0 = wv & (kUnmasked - 1);
-        const uint64_t pm = PM[x];
-        // up to kRegPreds predecessors are loaded into registers once, and the
-        // passes of the gap search then read no memory
-        constexpr int kRegPreds = 8;
-        const bool in_regs = !(wv & kUnmasked) && __popcll(pm) <= kRegPreds;
-        W ro[kRegPreds], re[kRegPreds];
-        if (in_regs) {
-            uint64_t m = pm;
-#pragma unroll
-            for (int j = 0; j < kRegPreds; ++j) {
-                ro[j] = 0;
-                re[j] = 0;  // an empty interval [0, 0) never conflicts and never raises the top
-                if (m) {
-                    const int32_t q = w0 + __ffsll((long long)m) - 1;
-                    m &= m - 1;
-                    ro[j] = OFFP[q];
-                    re[j] = (W)(ro[j] + AR[q].s);
-                }
-            }
+        const int32_t x = xn;
+        const ARec<I, W> me = men;
+        const int32_t wv = wvn;
+        const uint64_t pm = pmn;
+        if (r + 1 < c) {
+            xn = ord[r + 1];
+            men = AR[xn];
+            wvn = W0[xn];
+            pmn = PM[xn];
         }
-        auto each = [&](auto&& fn) {
-            if (in_regs) {
-#pragma unroll
-                for (int j = 0; j < kRegPreds; ++j) fn(ro[j], re[j]);
-            } else if (!(wv & kUnmasked)) {
-                for (uint64_t m = pm; m; m &= m - 1) {
-                    const int32_t q = w0 + __ffsll((long long)m) - 1;
-                    const W o = OFFP[q];
-                    fn(o, (W)(o + AR[q].s));
+        const int32_t w0 = wv & (kUnmasked - 1);
+        W o;
+        if (!(wv & kUnmasked)) {
+            // this lane's predecessors: window positions lane and lane + 32
+            const bool h1 = (pm >> lane) & 1ull, h2 = (pm >> (lane + 32)) & 1ull;
+            W o1 = 0, e1 = 0, o2 = 0, e2 = 0;  // an empty [0, 0) never conflicts
+            if (h1) {
+                o1 = voff[w0 + lane];
+                e1 = (W)(o1 + AR[w0 + lane].s);
+            }
+            if (h2) {
+                o2 = voff[w0 + lane + 32];
+                e2 = (W)(o2 + AR[w0 + lane + 32].s);
+            }
+            auto each = [&](auto&& fn) {
+                fn(o1, e1);
+                fn(o2, e2);
+            };
+            if (policy == MP_FIT_FIRST) {
+                o = 0;
+                for (;;) {
+                    W hit = 0;
+                    each([&](W po, W pe) {
+                        if (po < o + me.s && o < pe && pe > hit) hit = pe;
+                    });
+                    hit = warp_max_w(hit);
+                    if (hit <= o) break;
+                    o = hit;
                 }
             } else {
-                const int32_t w1 = min(p0 + c, BEND[(int32_t)me.f - 1]);
-                for (int32_t q = w0; q < w1; ++q) {
+                o = warp_best_fit<W>(me.s, each);
+            }
+        } else {  // a window too wide for a mask: its candidates tested on every pass
+            const int32_t w1 = min(p0 + c, BEND[(int32_t)me.f - 1]);
+            auto each = [&](auto&& fn) {
+                for (int32_t q = w0 + lane; q < w1; q += 32) {
                     if (q == x) continue;
                     const ARec<I, W> oq = AR[q];
                     if ((int32_t)oq.a < (int32_t)me.f && (int32_t)me.a < (int32_t)oq.f && precedes(oq, me)) {
-                        const W o = OFFP[q];
-                        fn(o, (W)(o + oq.s));
+                        const W po = voff[q];
+                        fn(po, (W)(po + oq.s));
                     }
                 }
+            };
+            if (policy == MP_FIT_FIRST) {
+                o = 0;
+                for (;;) {
+                    W hit = 0;
+                    each([&](W po, W pe) {
+                        if (po < o + me.s && o < pe && pe > hit) hit = pe;
+                    });
+                    hit = warp_max_w(hit);
+                    if (hit <= o) break;
+                    o = hit;
+                }
+            } else {
+                o = warp_best_fit<W>(me.s, each);
             }
-        };
-        W o;
-        if (policy == MP_FIT_FIRST) {
-            o = fit_first_scan<W>(me.s, each);
-        } else {
-            W top = 0;
-            each([&](W, W pe) { top = pe > top ? pe : top; });
-            o = fit_best_scan<W>(me.s, top, each);
         }
-        OFFP[x] = o;
+        if (lane == 0) voff[x] = o;
+        __syncwarp();
         mx = o + me.s > mx ? o + me.s : mx;
     }
     return mx;
@@ -1078,9 +1145,10 @@ __device__ W walk_comp(const ARec<I, W>* AR, W* OFFP, const int32_t* BEND, const
 // Places the nx large components starting at LST[0, nx) (the 32-bit launch
 // defers traces with components above kDeferComp, and with its data in the
 // workspace, every trace that needs this tier).  Each is first sorted into
-// priority order by the whole CTA.  Components whose members all live at most
-// kLongLife steps are then placed concurrently, one thread walking each
-// (walk_comp).  In the others the long-lived members cut the priority
+// priority order by the whole CTA.  Components of more than kWalkMin members
+// that all live at most kLongLife steps are then placed concurrently, one
+// warp walking each (walk_comp).  In the others the long-lived members (if
+// any) cut the priority
 // order into runs of short-lived ones, which the warps place together from a
 // ready queue, each long-lived one then by the whole CTA.  Returns this
 // thread's largest end.
@@ -1112,11 +1180,12 @@ __device__ __forceinline__ W large_tier(const ARec<I, W>* AR, W* OFFP, const int
         for (int32_t r = threadIdx.x; r < sz; r += blockDim.x) ORD[p0 + r] = sortbuf[r];
     }
     __syncthreads();
-    // 2. components without long-lived members.  First the whole CTA gives
+    // 2. components of more than kWalkMin members without long-lived ones.  First the whole CTA gives
     // every member its window and the mask of its predecessors there (W0
     // aliases HR, PM the CNT and QUE words, both free until step 3; W0[p0] = -1
-    // marks a component left to step 3); then one thread walks each component,
+    // marks a component left to step 3); then one warp walks each component,
     // all components at once.
+    {
     int32_t* W0 = HR;
     uint64_t* PM = reinterpret_cast<uint64_t*>(CNT);
     for (int32_t qc = 0; qc < nx; ++qc) {
@@ -1127,7 +1196,7 @@ __device__ __forceinline__ W large_tier(const ARec<I, W>* AR, W* OFFP, const int
             any_long |= life > kLongLife ? 1 : 0;
             if (life <= kLongLife) lw = max(lw, life);
         }
-        if (__syncthreads_or(any_long)) {
+        if (__syncthreads_or(any_long) || sz <= kWalkMin) {
             if (threadIdx.x == 0) W0[p0] = -1;
             continue;
         }
@@ -1152,19 +1221,17 @@ __device__ __forceinline__ W large_tier(const ARec<I, W>* AR, W* OFFP, const int
         }
     }
     __syncthreads();
-    {
-        const int lane = threadIdx.x & 31;
-        for (int32_t qc = warp + nwarps * lane; qc < nx; qc += blockDim.x) {
-            const int32_t p0 = LST[qc];
-            if (W0[p0] < 0) continue;
-            const W e = walk_comp<I, W>(AR, OFFP, BEND, ORD + p0, W0, PM, p0, comp_size(SB, NW, p0, n), policy);
-            mx = max(mx, e);
-        }
+    for (int32_t qc = warp; qc < nx; qc += nwarps) {  // a warp per component
+        const int32_t p0 = LST[qc];
+        if (W0[p0] < 0) continue;
+        const W e = walk_comp<I, W>(AR, OFFP, BEND, ORD + p0, W0, PM, p0, comp_size(SB, NW, p0, n), policy);
+        mx = max(mx, e);
     }
     __syncthreads();
-    // 3. components with long-lived members, one after the other: their
-    // long-lived members cut the priority order into runs of short-lived ones,
-    // which the warps place together, each long-lived one then by the whole CTA
+    }
+    // 3. the other components, one after the other: their long-lived members
+    // (if any) cut the priority order into runs of short-lived ones, which the
+    // warps place together, each long-lived one then by the whole CTA
     for (int32_t qc = 0; qc < nx; ++qc) {
         const int32_t p0 = LST[qc];
         const int32_t sz = comp_size(SB, NW, p0, n);
@@ -1194,7 +1261,7 @@ __device__ __forceinline__ W large_tier(const ARec<I, W>* AR, W* OFFP, const int
             }
             nl += tot;
         }
-        if (nl == 0) continue;  // placed in step 2 (nl is the block total: the same in every thread)
+        if (nl == 0 && sz > kWalkMin) continue;  // walked in step 2 (nl: a block total, uniform)
         __syncthreads();
         int64_t lw_max;
         block_excl_max((int64_t)lw, red, &lw_max);
