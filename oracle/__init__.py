@@ -8,8 +8,9 @@ library.  Every function takes a ``tracegen.TraceSet`` (host numpy arrays).
 Passages followed: Eq. 2.1 with its pairwise ordering constraints and the
 strategy list of Sec. 2.3 (greedy_by_size, bump_allocation); Sec. 3.2 makes
 greedy_by_size the default; Sec. 6 describes greedy by breadth (operators by
-the sizes of their tensors), read here with the operator at step t using the
-tensors live at t.
+the sizes of their input and output tensors), read here with the operator at
+step t producing the tensors allocated at t and using for the last time the
+tensors freed at t + 1.
 """
 from __future__ import annotations
 
@@ -112,7 +113,7 @@ def plan_greedy_by_size(ts, policy: int = FIT_FIRST):
 
 
 def plan_greedy_by_breadth(ts, policy: int = FIT_FIRST):
-    """Greedy by breadth (operator at step t = the tensors live at t): returns
+    """Greedy by breadth (operator at step t: outputs allocated at t, inputs last used at t): returns
     (offsets int64[N], plan_peak int64[B], status int32[B])."""
     lib, keep = _load(), []
     ref, _b = _batch(ts, keep)

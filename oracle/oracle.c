@@ -210,8 +210,8 @@ OR_EXPORT int or_plan_greedy_by_size(const or_batch *B, int32_t policy, int64_t 
 
 /* ------------------------------------------------------ greedy by breadth */
 
-static const int64_t *g_m;  /* per tensor: the largest live bytes over its lifetime */
-static const int32_t *g_t;  /* per tensor: the first step at which that is reached */
+static const uint64_t *g_m; /* per tensor: the larger breadth of its two operators */
+static const int32_t *g_t;  /* per tensor: the step of that operator (the earlier on ties) */
 
 /* Breadth order: the widest operator first (earlier step on ties), then the
  * greedy_by_size priority inside an operator. */
@@ -241,21 +241,27 @@ OR_EXPORT int or_plan_greedy_by_breadth(const or_batch *B, int32_t policy, int64
             continue;
         }
         int32_t T = B->steps[b];
-        /* operator t's breadth: the bytes of the tensors live at t */
-        int64_t *breadth = (int64_t *)calloc((size_t)(T > 0 ? T : 1), sizeof(int64_t));
-        for (int32_t i = 0; i < n; ++i)
-            for (int32_t t = a[i]; t < f[i]; ++t) breadth[t] += s[i];
+        /* The operator at step t produces the tensors allocated at t and uses
+         * for the last time the tensors freed at t + 1: its breadth is the
+         * bytes of both (a tensor of one step counts once).  Every tensor
+         * counts for at most two operators, so a breadth stays below 2^64. */
+        uint64_t *breadth = (uint64_t *)calloc((size_t)(T > 0 ? T : 1), sizeof(uint64_t));
+        for (int32_t i = 0; i < n; ++i) {
+            breadth[a[i]] += (uint64_t)s[i];
+            if (f[i] - 1 != a[i]) breadth[f[i] - 1] += (uint64_t)s[i];
+        }
         const size_t cap = (size_t)(n > 0 ? n : 1);
-        int64_t *m = (int64_t *)malloc(sizeof(int64_t) * cap);
+        uint64_t *m = (uint64_t *)malloc(sizeof(uint64_t) * cap);
         int32_t *tm = (int32_t *)malloc(sizeof(int32_t) * cap);
         int32_t *order = (int32_t *)malloc(sizeof(int32_t) * cap);
         for (int32_t i = 0; i < n; ++i) {
-            m[i] = -1;
-            for (int32_t t = a[i]; t < f[i]; ++t)
-                if (breadth[t] > m[i]) {
-                    m[i] = breadth[t];
-                    tm[i] = t;
-                }
+            /* a tensor is placed by the wider of its producer and its last user */
+            m[i] = breadth[a[i]];
+            tm[i] = a[i];
+            if (breadth[f[i] - 1] > m[i]) {
+                m[i] = breadth[f[i] - 1];
+                tm[i] = f[i] - 1;
+            }
             order[i] = i;
         }
         g_a = a;

@@ -45,13 +45,17 @@ int or_live_profile(const or_batch *b, int64_t *profile, int64_t *peak_lb, int32
 int or_plan_greedy_by_size(const or_batch *b, int32_t policy, int64_t *offsets, int64_t *plan_peak,
                            int32_t *trace_status);
 
-/* Greedy by breadth (the strategy of Pisarchyk et al. discussed in Sec. 6),
- * read for traces without operator records: the operator at step t uses the
- * tensors live at t, so its breadth is the live bytes at t.  Operators are
- * taken by breadth descending (earlier step on ties), each taking its not yet
- * placed tensors by the greedy_by_size priority; so a tensor's place in the
- * order is the widest operator over its lifetime, then size desc, alloc asc,
- * id asc.  Placement as greedy_by_size with the given policy. */
+/* Greedy by breadth (the strategy of Pisarchyk et al. discussed in Sec. 6):
+ * operators by breadth -- the sizes of their input and output tensors --
+ * descending.  A trace has one operator per step and no consumer lists, so
+ * the operator at step t is read as producing the tensors allocated at t
+ * (outputs) and using for the last time the tensors freed at t + 1 (inputs);
+ * its breadth is the bytes of both, a tensor of one step counting once.
+ * Operators are taken by breadth descending (earlier step on ties), each
+ * taking its not yet placed tensors by the greedy_by_size priority; so a
+ * tensor's place in the order is the wider of its producer and its last user,
+ * then size desc, alloc asc, id asc.  Placement as greedy_by_size with the
+ * given policy. */
 int or_plan_greedy_by_breadth(const or_batch *b, int32_t policy, int64_t *offsets, int64_t *plan_peak,
                               int32_t *trace_status);
 

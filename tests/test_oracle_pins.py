@@ -303,15 +303,32 @@ def test_breadth_hand_case_orders_by_the_widest_operator():
     assert list(off_s) == [20, 0, 4, 8, 12, 16, 25, 0] and pk_s[0] == 29
 
 
-def test_breadth_equals_size_when_every_tensor_spans_the_widest_step():
-    # every lifetime contains step 3, the widest one: one operator, size order
+def test_breadth_reads_operators_by_their_inputs_and_outputs():
+    """T = 3, tensors (alloc, free, size): t0 (2, 3, 12), t1 (0, 3, 10), t2
+    (1, 2, 9), t3 (0, 2, 3), t4 (0, 3, 8).  Operator 0 produces t1, t3, t4
+    (21 bytes); operator 1 produces t2 and uses t3 last (12); operator 2
+    produces t0 and uses t1 and t4 last (30).  So t0, t1, t4 go first (operator
+    2, by size), then t3 (operator 0), then t2 (operator 1).  FIRST: t0 at 0,
+    t1 above it at 12, t4 above both at 22, t3 at 0 (it meets t1 and t4 only),
+    t2 at 3 (above t3, below t1): peak 30.  Reading an operator as every
+    tensor live at its step would make operators 1 and 2 tie at 30 bytes and
+    give [27, 0, 10, 27, 19]; greedy_by_size gives [0, 12, 0, 9, 22]."""
+    ts = tg.from_tuples([(3, [(2, 3, 12), (0, 3, 10), (1, 2, 9), (0, 2, 3), (0, 3, 8)])])
+    off, pk, st = oracle.plan_greedy_by_breadth(ts, oracle.FIT_FIRST)
+    assert st[0] == 0 and list(off) == [0, 12, 3, 0, 22] and pk[0] == 30
+    off_s, _, _ = oracle.plan_greedy_by_size(ts, oracle.FIT_FIRST)
+    assert list(off_s) == [0, 12, 0, 9, 22]
+
+
+def test_breadth_equals_size_when_one_operator_produces_everything():
+    # every tensor is allocated at step 0: operator 0 produces all of them and
+    # is at least as wide as any last user, so the order is the size order
     rng = np.random.default_rng(11)
     for _ in range(20):
         n = int(rng.integers(1, 12))
-        a = rng.integers(0, 4, n)
-        f = rng.integers(4, 8, n)
+        f = rng.integers(1, 8, n)
         s = rng.integers(1, 100, n)
-        ts = tg.from_tuples([(8, list(zip(a, f, s)))])
+        ts = tg.from_tuples([(8, [(0, int(f[k]), int(s[k])) for k in range(n)])])
         for pol in (oracle.FIT_FIRST, oracle.FIT_BEST):
             assert np.array_equal(oracle.plan_greedy_by_breadth(ts, pol)[0], oracle.plan_greedy_by_size(ts, pol)[0])
 
