@@ -274,13 +274,15 @@ mp_status mp_plan_bump(const mp_batch *batch, int64_t *offsets, int64_t *plan_pe
 size_t mp_breadth_workspace_bytes(const mp_batch *batch);
 
 /* Greedy by breadth, the strategy of Pisarchyk et al. discussed in Sec. 6:
- * operators in order of breadth (the sizes of the tensors they use)
- * descending, each assigning offsets to its tensors not yet placed, largest
- * first, with greedy_by_size's gap search (policy as for
- * mp_plan_greedy_by_size).  Traces carry no operator records, so the operator
- * at step t is read as using the tensors live at t (breadth = live bytes at
- * t; ties: the earlier step first): a tensor is placed with the widest
- * operator over its lifetime.
+ * operators in order of breadth (the sizes of their input and output
+ * tensors) descending, each assigning offsets to its tensors not yet placed,
+ * largest first, with greedy_by_size's gap search (policy as for
+ * mp_plan_greedy_by_size).  A trace has one operator per step and no consumer
+ * lists, so the operator at step t is read as producing the tensors allocated
+ * at t and using for the last time the tensors freed at t + 1: its breadth is
+ * the bytes of both, a tensor of one step counting once (ties: the earlier
+ * step first), and a tensor is placed with the wider of its producer and its
+ * last user.
  * offsets, plan_peak, trace_status as for mp_plan_greedy_by_size (a failed
  * trace gets plan_peak 0).  workspace: at least
  * mp_breadth_workspace_bytes(batch) bytes, rules as for

@@ -235,8 +235,9 @@ def plan_bump(batch: DeviceBatch, offsets=None, plan_peak=None, status=None, wor
 
 def plan_greedy_by_breadth(batch: DeviceBatch, policy="first", offsets=None, plan_peak=None, status=None,
                            workspace: "Workspace | None" = None, stream=None):
-    """Greedy by breadth (Sec. 6; the operator at step t uses the tensors live
-    at t).  Returns (offsets, plan_peak, status)."""
+    """Greedy by breadth (Sec. 6; the operator at step t produces the tensors
+    allocated at t and uses last the tensors freed at t + 1).  Returns
+    (offsets, plan_peak, status)."""
     lib, dev = _lib.load(), batch.device
     offsets = _empty(batch.n_tensors, torch.int64, dev) if offsets is None else offsets
     plan_peak = _empty(batch.n_traces, torch.int64, dev) if plan_peak is None else plan_peak

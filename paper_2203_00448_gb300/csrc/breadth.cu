@@ -1,15 +1,17 @@
 // breadth.cu -- greedy by breadth, the strategy of Pisarchyk et al. that
-// Sec. 6 discusses: operators are taken by breadth (the sizes of the tensors
-// they use) descending, and each assigns offsets to its tensors not yet
-// placed, largest first, by greedy_by_size's gap search.  Traces carry no
-// operator records, so the operator at step t is read as using the tensors
-// live at t: its breadth is the live bytes at t, and a tensor is placed by
-// the widest operator over its lifetime.  The order is therefore: widest
-// breadth over the lifetime descending, the first step reaching it, then size
-// descending, alloc step ascending, id ascending.
+// Sec. 6 discusses: operators are taken by breadth (the sizes of their input
+// and output tensors) descending, and each assigns offsets to its tensors not
+// yet placed, largest first, by greedy_by_size's gap search.  A trace has one
+// operator per step and no consumer lists, so the operator at step t is read
+// as producing the tensors allocated at t and using for the last time the
+// tensors freed at t + 1: its breadth is the bytes of both (a tensor of one
+// step counts once), and a tensor is placed by the wider of its producer and
+// its last user.  The order is therefore: that breadth descending, that
+// operator's step (the earlier on ties), then size descending, alloc step
+// ascending, id ascending.
 //
-// GPU form: one CTA per trace.  The live profile (difference array and
-// scan), each tensor's widest step (a pass over its lifetime), an in-place
+// GPU form: one CTA per trace.  The breadths (two integer atomics per
+// tensor, order-independent), each tensor's wider operator, an in-place
 // odd-even merge sort of the ids by that order, then placement tensor by
 // tensor: all warps gather the placed tensors whose lifetimes overlap the
 // next one (one shared counter update per warp) and warp 0 runs the gap
@@ -21,8 +23,8 @@ namespace mp {
 
 namespace {
 
-// Per-trace working set: live bytes per step; per tensor (by id) its widest
-// breadth and step, (alloc, free), size and offset; the priority order; the
+// Per-trace working set: the breadth of the operator at each step; per tensor
+// (by id) its operator's breadth and step, (alloc, free), size and offset; the priority order; the
 // gathered predecessors' offsets and ends.
 struct BreadthLayout {
     size_t prof, km, kt, ord, af, sz, off, pb, pe, total;
@@ -173,8 +175,10 @@ k_breadth(mp_batch bt, int32_t policy, int64_t* __restrict__ offsets, int64_t* _
         AF[k] = make_int2(a, f);
         SZ[k] = s;
         ORD[k] = k;
+        // outputs of the operator at a, inputs of the operator at f - 1 (a
+        // tensor counts for two operators at most: the sums stay below 2^64)
         atomic_add_u64_split(PROF + a, (uint64_t)s);
-        if (f < T) atomic_add_u64_split(PROF + f, (uint64_t)(-s));
+        if (f - 1 != a) atomic_add_u64_split(PROF + (f - 1), (uint64_t)s);
     }
     block_add_size_sum(sum, &s_hi, &s_lo);
     if (bad) s_bad = 1;
@@ -186,24 +190,24 @@ k_breadth(mp_batch bt, int32_t policy, int64_t* __restrict__ offsets, int64_t* _
         }
         return;
     }
-    block_incl_scan_max_i64<8>(PROF, T, 0, red);  // PROF[t] = the live bytes at t: operator t's breadth
-
-    // each tensor's widest operator: the largest breadth over its lifetime, first step reaching it
+    // PROF[t] (as uint64): the breadth of the operator at step t.  Each
+    // tensor's operator: the wider of its producer and its last user, the
+    // earlier one on ties
+    const uint64_t* BR = reinterpret_cast<const uint64_t*>(PROF);
     for (int k = threadIdx.x; k < n; k += blockDim.x) {
         const int2 af = AF[k];
-        int64_t m = -1;
+        uint64_t m = BR[af.x];
         int32_t tm = af.x;
-        for (int32_t t = af.x; t < af.y; ++t)
-            if (PROF[t] > m) {
-                m = PROF[t];
-                tm = t;
-            }
-        KM[k] = m;
+        if (BR[af.y - 1] > m) {
+            m = BR[af.y - 1];
+            tm = af.y - 1;
+        }
+        KM[k] = (int64_t)m;
         KT[k] = tm;
     }
     __syncthreads();
     block_sort_ids(ORD, n, [&](int32_t x, int32_t y) {
-        if (KM[x] != KM[y]) return KM[x] > KM[y];
+        if (KM[x] != KM[y]) return (uint64_t)KM[x] > (uint64_t)KM[y];
         if (KT[x] != KT[y]) return KT[x] < KT[y];
         if (SZ[x] != SZ[y]) return SZ[x] > SZ[y];
         if (AF[x].x != AF[y].x) return AF[x].x < AF[y].x;
