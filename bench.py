@@ -668,6 +668,8 @@ def run_all_configs(args):
     peak, peak_kind = measured_peaks()
     stream = torch.cuda.current_stream()
     for k in sorted(tracegen.CONFIG_NAMES):
+        if args.config is not None and k != args.config:
+            continue
         ts = tracegen.config(k)
         db = mp.DeviceBatch.from_host(ts, dev)
         buf = mp.PathBuffers(db)
@@ -685,8 +687,10 @@ def run_all_configs(args):
         ok = bool((buf.status[0] == 0).all()) and bool((buf.verdict == 1).all())
         ms = statistics.median(times)
         nbytes = algorithmic_bytes(FUSED, ts.n_tensors, ts.n_traces, ts.n_steps)
-        one_core = _oracle_path_seconds(ts)
-        all_cores, n_chunks = oracle_all_cores(ts, pool, cores)
+        one_core = all_cores = n_chunks = None
+        if args.oracle_traces > 0:  # 0: a profiling run, no oracle legs
+            one_core = _oracle_path_seconds(ts)
+            all_cores, n_chunks = oracle_all_cores(ts, pool, cores)
         gbs = nbytes / (ms * 1e-3) / 1e9
         print(json.dumps({
             "workload": tracegen.CONFIG_NAMES[k], "policy": args.policy, "ok": ok, "n_traces": ts.n_traces,
@@ -719,7 +723,10 @@ def main(argv=None):
     ap.add_argument("--traces", type=int, default=WORKLOAD["n_traces"],
                     help="traces per rank (the reported workload is the default 4096; other values are for profiling)")
     ap.add_argument("--all-configs", action="store_true",
-                    help="time every workload (one JSON line each) beside the oracle on 1 and on all host cores")
+                    help="time every workload (one JSON line each) beside the oracle on 1 and on all host cores "
+                         "(--oracle-traces 0 leaves the oracle out)")
+    ap.add_argument("--config", type=int, default=None,
+                    help="with --all-configs: that workload only (tracegen.CONFIG_NAMES)")
     args = ap.parse_args(argv)
     if args.all_configs:
         return run_all_configs(args)

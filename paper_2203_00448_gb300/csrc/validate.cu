@@ -19,9 +19,10 @@ namespace mp {
 
 namespace {
 
-// Per-trace working set: tensors scattered into alloc-step order as (offset,
-// end) records -- 8 bytes when every end of the trace is below 2^32, else 16
-// -- and (free step, id) pairs, plus the bucket ends.
+// Per-trace working set: tensors scattered into alloc-step order as 16-byte
+// records -- (offset, end, free step, id) as 32-bit words when every end of
+// the trace is below 2^32, else (offset, end) as 64-bit words with the (free
+// step, id) pairs beside them -- plus the bucket ends.
 struct ValidateLayout {
     size_t rec, fi, bend, total;
     __host__ __device__ ValidateLayout(int64_t n, int64_t T) {
@@ -109,23 +110,37 @@ __device__ void block_excl_scan_i32(int32_t* x, int32_t len, int32_t* red) {
     __syncthreads();
 }
 
+__device__ __forceinline__ unsigned long long pair_key(uint32_t i, uint32_t j) {
+    const uint32_t lo = i < j ? i : j, hi = i < j ? j : i;
+    return ((unsigned long long)lo << 32) | hi;
+}
+
 // Every lifetime-overlapping pair once, from its earlier member in alloc
-// order (positions p < q < BEND[f_p - 1]); records R are (offset, end).
-template <typename R>
-__device__ __forceinline__ void check_pairs(const R* __restrict__ rec, const int2* __restrict__ fi_arr,
-                                            const int32_t* __restrict__ bend, int32_t n, unsigned long long* key) {
+// order (positions p < q < BEND[f_p - 1]), over narrow records.
+__device__ __forceinline__ void check_pairs_narrow(const uint4* __restrict__ rec, const int32_t* __restrict__ bend,
+                                                   int32_t n, unsigned long long* key) {
+    for (int32_t p = threadIdx.x; p < n; p += blockDim.x) {
+        const uint4 ri = rec[p];
+        const int32_t stop = bend[(int32_t)ri.z - 1];
+        for (int32_t q = p + 1; q < stop; ++q) {
+            const uint4 rj = rec[q];
+            if (ri.x < rj.y && rj.x < ri.y) atomicMin(key, pair_key(ri.w, rj.w));
+        }
+    }
+}
+
+// The same over 64-bit (offset, end) records with the (free step, id) pairs beside them.
+__device__ __forceinline__ void check_pairs_wide(const longlong2* __restrict__ rec, const int2* __restrict__ fi_arr,
+                                                 const int32_t* __restrict__ bend, int32_t n,
+                                                 unsigned long long* key) {
     for (int32_t p = threadIdx.x; p < n; p += blockDim.x) {
         const int2 fi = fi_arr[p];
         const int32_t stop = bend[fi.x - 1];
         if (stop <= p + 1) continue;
-        const R ri = rec[p];
+        const longlong2 ri = rec[p];
         for (int32_t q = p + 1; q < stop; ++q) {
-            const R rj = rec[q];
-            if (ri.x < rj.y && rj.x < ri.y) {
-                const uint32_t i = (uint32_t)fi.y, j = (uint32_t)fi_arr[q].y;
-                const uint32_t lo = i < j ? i : j, hi = i < j ? j : i;
-                atomicMin(key, ((unsigned long long)lo << 32) | hi);
-            }
+            const longlong2 rj = rec[q];
+            if (ri.x < rj.y && rj.x < ri.y) atomicMin(key, pair_key((uint32_t)fi.y, (uint32_t)fi_arr[q].y));
         }
     }
 }
@@ -207,17 +222,18 @@ k_validate(mp_batch bt, const int64_t* __restrict__ offsets, int32_t* __restrict
     // Checks, flags and the alloc-step histogram.  The cached tensors keep
     // their offset and end as 32-bit words from here on (all the narrow path
     // needs); the wide path and the exact size sum read memory again.
-    int flags = 0;
+    uint32_t bad = 0;
+    uint64_t or_e = 0, or_s = 0;
+    // (0 <= a < f <= T as two unsigned compares, T being >= 0; the flags are
+    // or-ed over the thread's tensors and read once.  An invalid tensor's
+    // bits are garbage there, but its trace fails with MP_EINVAL anyway.)
     auto take = [&](int32_t a, int32_t f, int64_t sz, int64_t o) -> uint64_t {
-        if (!tensor_ok(a, f, sz, T) || o < 0) {
-            flags |= kFlagInvalid;
-            return 0;
-        }
-        const uint64_t e = (uint64_t)o + (uint64_t)sz;  // both below 2^63: no wrap
-        flags |= (e >> 63) ? kFlagEndOvf : 0;
-        flags |= (e >> 32) ? kFlagWide : 0;
-        flags |= ((uint64_t)sz >> 32) ? kFlagBigSize : 0;
-        atomicAdd(BEND + a, 1);
+        const bool ok = (uint32_t)a < (uint32_t)f && (uint32_t)f <= (uint32_t)T && sz > 0 && o >= 0;
+        const uint64_t e = (uint64_t)o + (uint64_t)sz;  // both below 2^63 when ok: no wrap
+        bad |= ok ? 0u : 1u;
+        or_e |= e;
+        or_s |= (uint64_t)sz;
+        if (ok) atomicAdd(BEND + a, 1);
         return e;
     };
     uint32_t co32[kValCached], ce32[kValCached];
@@ -228,6 +244,8 @@ k_validate(mp_batch bt, const int64_t* __restrict__ offsets, int32_t* __restrict
     }
     const int32_t nc = min(n, kValCached * nthr);
     for (int32_t k = nc + tid; k < n; k += nthr) take(__ldg(Ag + k), __ldg(Fg + k), __ldg(Sg + k), __ldg(Og + k));
+    int flags = (bad ? kFlagInvalid : 0) | ((or_e >> 63) ? kFlagEndOvf : 0) | ((or_e >> 32) ? kFlagWide : 0) |
+                ((or_s >> 32) ? kFlagBigSize : 0);
     flags = (int)__reduce_or_sync(0xffffffffu, (unsigned)flags);
     if ((tid & 31) == 0 && flags) atomicOr(&sh.flags, flags);
     __syncthreads();
@@ -252,17 +270,17 @@ k_validate(mp_batch bt, const int64_t* __restrict__ offsets, int32_t* __restrict
     // BEND[t] is the end of bucket t (tensors with alloc <= t).
     block_excl_scan_i32(BEND, T, red);
     const bool wide = (F & kFlagWide) != 0;
-    uint2* REC32 = reinterpret_cast<uint2*>(base + L.rec);
+    uint4* REC32 = reinterpret_cast<uint4*>(base + L.rec);
     longlong2* REC64 = reinterpret_cast<longlong2*>(base + L.rec);
     auto scatter = [&](int32_t k, int32_t a, int32_t f, uint32_t o32, uint32_t e32) {
         const int32_t pos = atomicAdd(BEND + a, 1);
         if (wide) {
             const int64_t o = __ldg(Og + k);
             REC64[pos] = make_longlong2(o, o + __ldg(Sg + k));
+            FI[pos] = make_int2(f, k);
         } else {
-            REC32[pos] = make_uint2(o32, e32);
+            REC32[pos] = make_uint4(o32, e32, (uint32_t)f, (uint32_t)k);
         }
-        FI[pos] = make_int2(f, k);
     };
 #pragma unroll
     for (int j = 0; j < kValCached; ++j) {
@@ -276,9 +294,9 @@ k_validate(mp_batch bt, const int64_t* __restrict__ offsets, int32_t* __restrict
     __syncthreads();
 
     if (wide)
-        check_pairs(REC64, FI, BEND, n, &sh.key);
+        check_pairs_wide(REC64, FI, BEND, n, &sh.key);
     else
-        check_pairs(REC32, FI, BEND, n, &sh.key);
+        check_pairs_narrow(REC32, BEND, n, &sh.key);
     __syncthreads();
     if (tid == 0) {
         const unsigned long long key = sh.key;
