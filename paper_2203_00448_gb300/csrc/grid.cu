@@ -683,8 +683,121 @@ __device__ __forceinline__ int64_t cta_excl_max(int64_t v, int64_t* red, int64_t
     return r;
 }
 
-constexpr int32_t kJumpCap = 128;  // FIRST jumps at most this often before it sorts instead
+constexpr int32_t kJumpCap = 128;  // FIRST jumps (no merge sort) at most this often before it sorts records
 constexpr int kRegJump = 6;        // predecessor pairs per thread held in registers for the jumps
+constexpr int kKeyIdxBits = 13;    // the merge sort's keys: offset << 13 | pair index
+constexpr int32_t kMergeMaxPairs = 1 << kKeyIdxBits;
+
+// Ascending bitonic network over a thread's E keys (all indices compile-time).
+template <int E>
+__device__ __forceinline__ void sort_regs(uint64_t (&k)[E]) {
+#pragma unroll
+    for (int kk = 2; kk <= E; kk <<= 1) {
+#pragma unroll
+        for (int j = kk >> 1; j > 0; j >>= 1) {
+#pragma unroll
+            for (int i = 0; i < E; ++i) {
+                const int l = i ^ j;
+                if (l > i) {
+                    const uint64_t a = k[i], b = k[l];
+                    const uint64_t lo = a < b ? a : b, hi = a < b ? b : a;
+                    const bool up = (i & kk) == 0;
+                    k[i] = up ? lo : hi;
+                    k[l] = up ? hi : lo;
+                }
+            }
+        }
+    }
+}
+
+// The merge sort's buffer: one 8-byte word of padding after every 16, so that
+// lanes reading or writing words E apart (E <= 16) fall in distinct banks.
+__device__ __forceinline__ int32_t mpad(int32_t i) { return i + (i >> 4); }
+
+// The sorted gap search of a CTA item over its P <= E * blockDim predecessor
+// pairs (offset, end) in the region, every offset below 2^(63 - kKeyIdxBits),
+// by a merge sort of 64-bit keys (offset << kKeyIdxBits | pair index).  The
+// keys are read in E chunks of blockDim pairs; each chunk's ends are then
+// packed at the region's start (8 bytes per pair: they only overwrite pairs of
+// earlier chunks, read before the chunk's barrier).  Each thread sorts its E
+// keys in registers; then log2(blockDim) rounds merge runs of doubling length
+// through a padded buffer behind the ends, each thread finding where its E
+// outputs start by a merge-path search.  A final scan over the sorted keys
+// exposes every gap as in the record sort.
+template <int E>
+__device__ int64_t merge_sort_fit(int64_t* region, int32_t P, int64_t s, int32_t policy, int64_t* red) {
+    const int32_t t = (int32_t)threadIdx.x, nt = (int32_t)blockDim.x;
+    const int32_t plen = E * nt;
+    int64_t* ends = region;  // [0, P) once packed
+    uint64_t* buf = reinterpret_cast<uint64_t*>(region + kMergeMaxPairs);
+    uint64_t k[E];
+#pragma unroll
+    for (int c = 0; c < E; ++c) {
+        const int32_t idx = c * nt + t;
+        int64_t en = 0;
+        k[c] = ~0ull;  // padding sorts last
+        if (idx < P) {
+            k[c] = ((uint64_t)region[2 * idx] << kKeyIdxBits) | (uint64_t)idx;
+            en = region[2 * idx + 1];
+        }
+        __syncthreads();
+        if (idx < P) ends[idx] = en;
+    }
+    sort_regs<E>(k);
+    for (int32_t L = E; L < plen; L <<= 1) {
+#pragma unroll
+        for (int e = 0; e < E; ++e) buf[mpad(t * E + e)] = k[e];
+        __syncthreads();
+        const int32_t d = (t * E) & (2 * L - 1);  // my first output within my merged run
+        const int32_t a0 = t * E - d, b0 = a0 + L;
+        int32_t lo = max(0, d - L), hi = min(d, L);
+        while (lo < hi) {  // how many of my run's first d outputs come from A (B first on ties)
+            const int32_t mid = (lo + hi) >> 1;
+            if (buf[mpad(a0 + mid)] < buf[mpad(b0 + d - 1 - mid)]) lo = mid + 1;
+            else hi = mid;
+        }
+        int32_t i = lo, j = d - lo;
+        uint64_t a = i < L ? buf[mpad(a0 + i)] : ~0ull, b = j < L ? buf[mpad(b0 + j)] : ~0ull;
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+            if (a < b) {
+                k[e] = a;
+                ++i;
+                a = i < L ? buf[mpad(a0 + i)] : ~0ull;
+            } else {
+                k[e] = b;
+                ++j;
+                b = j < L ? buf[mpad(b0 + j)] : ~0ull;
+            }
+        }
+        __syncthreads();
+    }
+    // thread t holds sorted positions [t E, t E + E): the gap before position
+    // p is its offset minus the largest end before it
+    int64_t local = 0;
+#pragma unroll
+    for (int e = 0; e < E; ++e)
+        if (t * E + e < P) local = max(local, ends[k[e] & (kMergeMaxPairs - 1)]);
+    int64_t top;
+    int64_t prev = cta_excl_max(local, red, &top);
+    int64_t key = INT64_MAX, val = INT64_MAX;
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+        if (t * E + e >= P) break;
+        const int64_t off = (int64_t)(k[e] >> kKeyIdxBits);
+        const int64_t gl = off - prev;
+        if (gl >= s) {
+            const int64_t kx = policy == MP_FIT_FIRST ? prev : gl;  // prev grows with the position
+            if (kx < key || (kx == key && prev < val)) {
+                key = kx;
+                val = prev;
+            }
+        }
+        prev = max(prev, ends[k[e] & (kMergeMaxPairs - 1)]);
+    }
+    block_min_pair(key, val, red);
+    return key == INT64_MAX ? top : val;
+}
 
 // Shared state of a CTA item.
 struct LongShared {
@@ -694,13 +807,15 @@ struct LongShared {
 // A tensor placed by the whole CTA (long-lived, or more predecessors than a
 // warp holds).  One pass over the candidates puts the predecessors' pairs in
 // the region (then in this CTA's overflow buffer, ovf) and lists the
-// successors after them (if too many, they are enumerated again).  FIRST jumps
-// to the largest conflicting end until nothing conflicts (pairs held in
-// registers, one block reduction per jump); if that takes more than kJumpCap
-// jumps, or for BEST, the pairs are sorted by offset and one scan exposes
-// every gap (FIRST: the lowest that fits; BEST: the smallest, the lowest on
-// ties).  Returns a successor that
-// became ready and is a CTA item, for this CTA to place next (-1 if none).
+// successors after them (if too many, they are enumerated again).  Up to
+// kMergeMaxPairs pairs with offsets below 2^(63 - kKeyIdxBits) are merge
+// sorted by offset (merge_sort_fit), and one scan exposes every gap (FIRST:
+// the lowest that fits; BEST: the smallest, the lowest on ties).  Otherwise
+// FIRST jumps to the largest conflicting end until nothing conflicts (pairs
+// held in registers, one block reduction per jump); if that takes more than
+// kJumpCap jumps, or for BEST, the (offset, end) records are sorted in memory
+// and scanned the same way.  Returns a successor that became ready and is a
+// CTA item, for this CTA to place next (-1 if none).
 __device__ int64_t place_long(const GridWs& w, const LongCache& lc, int64_t g, int32_t policy, int64_t* region,
                               int64_t* ovf, int64_t* red, LongShared* sh) {
     const Node x = load_node(w, g);
@@ -740,10 +855,12 @@ __device__ int64_t place_long(const GridWs& w, const LongCache& lc, int64_t g, i
     // the predecessors' offsets: every thread's loads in flight together; the
     // first kRegJump * blockDim pairs also stay in registers for the jumps
     int64_t ro[kRegJump], re[kRegJump];
+    uint64_t obits = 0;  // the or of this thread's offsets
 #pragma unroll
     for (int j = 0; j < kRegJump; ++j) {
         const int32_t k = (int32_t)threadIdx.x + j * stride;
         ro[j] = k < P ? off_of(w, pair_at(k)[0]) : 0;
+        obits |= (uint64_t)ro[j];
     }
 #pragma unroll
     for (int j = 0; j < kRegJump; ++j) {
@@ -770,13 +887,23 @@ __device__ int64_t place_long(const GridWs& w, const LongCache& lc, int64_t g, i
                 int64_t* q = pair_at(k);
                 q[1] += po[u];
                 q[0] = po[u];
+                obits |= (uint64_t)po[u];
             }
         }
     }
-    __syncthreads();
+    // whether some offset is too wide for the merge sort's keys
+    const bool wide_keys = __syncthreads_or((obits >> (63 - kKeyIdxBits)) != 0);
     int64_t o = 0;
-    bool sorted = policy == MP_FIT_BEST;
-    if (!sorted) {  // one barrier per jump: the warps' maxima alternate between two buffers
+    const int32_t nt = (int32_t)blockDim.x;
+    const bool merge = !wide_keys && P <= kMergeMaxPairs && P <= 16 * nt;
+    bool sorted = !merge && policy == MP_FIT_BEST;
+    if (merge) {
+        o = P <= nt       ? merge_sort_fit<1>(region, P, s, policy, red)
+            : P <= 2 * nt ? merge_sort_fit<2>(region, P, s, policy, red)
+            : P <= 4 * nt ? merge_sort_fit<4>(region, P, s, policy, red)
+            : P <= 8 * nt ? merge_sort_fit<8>(region, P, s, policy, red)
+                          : merge_sort_fit<16>(region, P, s, policy, red);
+    } else if (!sorted) {  // one barrier per jump: the warps' maxima alternate between two buffers
         const int lane = threadIdx.x & 31, wp = threadIdx.x >> 5;
         for (int32_t jumps = 0;; ++jumps) {
             if (jumps == kJumpCap) {

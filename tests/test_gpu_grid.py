@@ -136,3 +136,25 @@ def test_grid_many_long_lived_neighbours(cuda_lib, name, pol):
     o = oracle_run(ts, pol)
     assert_parity(ts, gpu_run(ts, name), o)
     _assert_fused(ts, _fused(ts, name), o)
+
+
+@pytest.mark.parametrize("name,pol", POLICIES)
+def test_grid_offsets_past_the_merge_keys(cuda_lib, name, pol):
+    """Sizes up to 2^45: offsets pass 2^50, beyond what the merge sort's 64-bit
+    keys hold next to a 13-bit pair index, so long-lived tensors fall back to
+    sorting (offset, end) records; a second trace of small sizes in the same
+    batch takes the merge sort."""
+    rng = np.random.default_rng(31)
+    traces = []
+    for big in (True, False):
+        n, T = 1600, 2400
+        a = rng.integers(0, T - 50, size=n)
+        life = np.where(rng.random(n) < 0.25, rng.integers(40, 1500, size=n), rng.integers(1, 8, size=n))
+        f = np.minimum(a + life, T)
+        s = rng.integers(1, 1 << 12, size=n) * ((1 << 33) if big else 16)
+        traces.append((T, a, f, s))
+    ts = tg.from_arrays(traces)
+    o = oracle_run(ts, pol)
+    assert (o["st"] == 0).all()
+    assert int(o["offsets"][: ts.trace_ptr[1]].max()) >= 1 << 50
+    assert_parity(ts, gpu_run(ts, name), o)
