@@ -599,3 +599,39 @@ def test_breadth_parity(cuda_lib, name, pol):
         for b in np.nonzero(o_st == 0)[0]:
             lo, hi = ts.trace_ptr[b], ts.trace_ptr[b + 1]
             assert np.array_equal(off[lo:hi], o_off[lo:hi]), (ts.name, b)
+
+
+@pytest.mark.parametrize("name,pol", POLICIES)
+def test_breadth_component_tiers(cuda_lib, name, pol):
+    """Greedy by breadth through its component kernel: components of 2..8
+    tensors (a thread each), 9..32 (a warp each) and larger (the whole CTA),
+    sizes drawn from two values so that breadths, steps and sizes tie often;
+    traces whose large components outgrow the CTA tier's scratch (more than
+    0.6 tensors per step) go to the per-tensor kernel in the same call."""
+    import paper_2203_00448_gb300 as mp
+
+    rng = np.random.default_rng(41)
+    traces = []
+    for b in range(300):
+        n, T = int(rng.integers(20, 400)), int(rng.integers(100, 900))
+        a = rng.integers(0, T - 1, size=n)
+        life = 1 + rng.geometric(0.35 if b % 7 else 0.08, size=n)
+        f = np.minimum(a + life, T)
+        s = rng.choice([64, 128], size=n)
+        traces.append((T, a, f, s))
+    ts = tg.from_arrays(traces)
+    big = 0
+    for b in range(ts.n_traces):
+        _, a, f, _ = ts.trace(b)
+        o = np.lexsort((np.arange(len(a)), a))
+        run = np.maximum.accumulate(np.asarray(f)[o])
+        starts = np.flatnonzero(np.r_[True, run[:-1] <= np.asarray(a)[o][1:]])
+        big += int(np.diff(np.r_[starts, len(a)]).max() > 32)
+    assert 0 < big < ts.n_traces
+    db = mp.DeviceBatch.from_host(ts, "cuda")
+    off, pk, st = mp.plan_greedy_by_breadth(db, name)
+    torch.cuda.synchronize()
+    o_off, o_pk, o_st = oracle.plan_greedy_by_breadth(ts, pol)
+    assert np.array_equal(st.cpu().numpy(), o_st) and (o_st == 0).all()
+    assert np.array_equal(pk.cpu().numpy(), o_pk)
+    assert np.array_equal(off.cpu().numpy(), o_off)
