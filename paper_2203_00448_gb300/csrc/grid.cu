@@ -801,7 +801,7 @@ __device__ int64_t merge_sort_fit(int64_t* region, int32_t P, int64_t s, int32_t
 
 // Shared state of a CTA item.
 struct LongShared {
-    int32_t np, ns, next;
+    int32_t np, ns;
 };
 
 // A tensor placed by the whole CTA (long-lived, or more predecessors than a
@@ -814,10 +814,11 @@ struct LongShared {
 // FIRST jumps to the largest conflicting end until nothing conflicts (pairs
 // held in registers, one block reduction per jump); if that takes more than
 // kJumpCap jumps, or for BEST, the (offset, end) records are sorted in memory
-// and scanned the same way.  Returns a successor that became ready and is a
-// CTA item, for this CTA to place next (-1 if none).
-__device__ int64_t place_long(const GridWs& w, const LongCache& lc, int64_t g, int32_t policy, int64_t* region,
-                              int64_t* ovf, int64_t* red, LongShared* sh) {
+// and scanned the same way.  Successors that become ready are queued, CTA
+// items too: an idle long CTA starts one while this one still drops the
+// others (keeping it for this CTA measured slower).
+__device__ void place_long(const GridWs& w, const LongCache& lc, int64_t g, int32_t policy, int64_t* region,
+                           int64_t* ovf, int64_t* red, LongShared* sh) {
     const Node x = load_node(w, g);
     const Cands c = cands_of(w, lc.lw[x.b], lc.nl[x.b], x);
     const int32_t ncand = (c.w1 - c.w0) + c.nlong;
@@ -826,7 +827,6 @@ __device__ int64_t place_long(const GridWs& w, const LongCache& lc, int64_t g, i
     if (threadIdx.x == 0) {
         sh->np = 0;
         sh->ns = 0;
-        sh->next = -1;
     }
     __syncthreads();
     auto pair_at = [&](int32_t k) -> int64_t* { return k < kRegionPairs ? region + 2 * k : ovf + 2 * (k - kRegionPairs); };
@@ -996,9 +996,7 @@ __device__ int64_t place_long(const GridWs& w, const LongCache& lc, int64_t g, i
     __threadfence();
     if (threadIdx.x == 0) atomicAdd(&w.ctl->placed, 1);
     auto ready = [&](int64_t slot) {
-        if (!drop(w, slot)) return;
-        if (slot != w.hold && cta_item(w, slot) && atomicCAS(&sh->next, -1, (int32_t)slot) == -1) return;
-        push(w, slot);
+        if (drop(w, slot)) push(w, slot);
     };
     if (S <= kLongSuccs) {  // the drops of a thread's successors in flight together
         for (int32_t k0 = threadIdx.x; k0 < S; k0 += 4 * stride) {
@@ -1014,7 +1012,6 @@ __device__ int64_t place_long(const GridWs& w, const LongCache& lc, int64_t g, i
             for (int u = 0; u < 4; ++u) {
                 if (old4[u] != 1) continue;
                 const int64_t slot = sl[u];
-                if (slot != w.hold && cta_item(w, slot) && atomicCAS(&sh->next, -1, (int32_t)slot) == -1) continue;
                 push(w, slot);
             }
         }
@@ -1029,10 +1026,7 @@ __device__ int64_t place_long(const GridWs& w, const LongCache& lc, int64_t g, i
                 if (sc[u] && !cand_precedes(w, x, cd[u])) ready(cd[u].slot);
         }
     }
-    __syncthreads();
-    const int64_t next = sh->next;
-    __syncthreads();
-    return next;
+    __syncthreads();  // every successor dropped before the region is reused
 }
 
 // Waits (bounded) until queue slot h (of the queue whose fill count is *tail)
@@ -1073,8 +1067,8 @@ __device__ int32_t take_slot(const GridWs& w, const int32_t* queue, const int32_
 // predecessors; then the first long_ctas CTAs place CTA items (thread 0 takes
 // the next long-queue slot for the whole CTA) and every warp of the others
 // places warp items (each takes the next short-queue slot for itself).  A
-// worker that makes a successor of its own kind ready places it next instead
-// of queueing it.  A worker waits only for the entry of the slot it took and
+// warp that makes a warp item ready places it next instead of queueing it; a
+// CTA queues every successor it makes ready.  A worker waits only for the entry of the slot it took and
 // never holds one entry while waiting for another; the lowest-ranked unplaced
 // tensor of a trace is always queued or being placed, so a taken slot is
 // always filled in the end.  With w.hold >= 0 (tests only) the tensor of that
@@ -1159,21 +1153,18 @@ k_grid_flow(mp_batch bt, int32_t policy, GridWs w, int32_t long_ctas) {
     const int32_t total = ctl->total;
     if ((int32_t)blockIdx.x < long_ctas) {
         int64_t* ovf = w.ovf_pairs > 0 ? w.ovf + (int64_t)blockIdx.x * 2 * w.ovf_pairs : nullptr;
-        int64_t next = -1;
         for (;;) {
-            if (next < 0) {
-                if (threadIdx.x == 0) {
-                    const int32_t h = atomicAdd(&ctl->head_l, 1);
-                    s_long = h < total ? take_slot(w, w.ql, &ctl->tail_l, h, total) : -1;
-                    __threadfence();  // the predecessors' offsets after the entry
-                }
-                __syncthreads();
-                next = s_long;
-                __syncthreads();
-                if (next < 0) break;
+            if (threadIdx.x == 0) {
+                const int32_t h = atomicAdd(&ctl->head_l, 1);
+                s_long = h < total ? take_slot(w, w.ql, &ctl->tail_l, h, total) : -1;
+                __threadfence();  // the predecessors' offsets after the entry
             }
+            __syncthreads();
+            const int64_t item = s_long;
+            __syncthreads();
+            if (item < 0) break;
             __threadfence();
-            next = place_long(w, lc, next, policy, region, ovf, red, &s_sh);
+            place_long(w, lc, item, policy, region, ovf, red, &s_sh);
         }
     } else {
         int64_t* buf = region + (int64_t)warp * (kWarpBytes / 8);
