@@ -211,7 +211,11 @@ size_t mp_host_path_bytes(const mp_batch *host_batch, int32_t chunks);
  * copy_in_stream, planned on compute_stream once they have landed, and its
  * profile and offsets copied back on copy_out_stream once planned, so the
  * copies of both directions overlap the planning of other runs; the
- * per-trace results follow the last run.  Page-locked (pinned) host memory
+ * per-trace results follow the last run.  The per-trace arrays move in one
+ * copy each way when the host keeps trace_ptr, profile_ptr and steps in this
+ * order with fewer than 16 bytes between them (read, never written), and
+ * peak_lb, plan_peak, verdict, conflict, trace_status adjacent in this order
+ * with no byte between them; otherwise one copy per array.  Page-locked (pinned) host memory
  * is needed for the copies to overlap; pageable memory is correct but
  * serialises them.  chunks = 0 stages nothing: the kernels read the inputs
  * from, and write the results to, the host arrays themselves over the

@@ -413,10 +413,14 @@ class HostPath:
         self.policy = policy
         dev = torch.device(device)
         B, N, S = int(ts.n_traces), int(ts.n_tensors), int(ts.n_steps)
-        in_specs = [("trace_ptr", (B + 1,), torch.int64), ("steps", (B,), torch.int32),
-                    ("profile_ptr", (B + 1,), torch.int64), ("alloc_step", (N,), torch.int32),
+        # the per-trace arrays in the orders mp_plan_and_validate_host moves in
+        # one copy each way: trace_ptr, profile_ptr, steps (at most 15 bytes
+        # apart); peak_lb, plan_peak, verdict, conflict, status (adjacent, which
+        # the 16-byte alignment of the packing keeps when B is a multiple of 4)
+        in_specs = [("trace_ptr", (B + 1,), torch.int64), ("profile_ptr", (B + 1,), torch.int64),
+                    ("steps", (B,), torch.int32), ("alloc_step", (N,), torch.int32),
                     ("free_step", (N,), torch.int32), ("size_bytes", (N,), torch.int64)]
-        out_specs = [("profile", (S,), torch.int64), ("peak_lb", (B,), torch.int64), ("offsets", (N,), torch.int64),
+        out_specs = [("profile", (S,), torch.int64), ("offsets", (N,), torch.int64), ("peak_lb", (B,), torch.int64),
                      ("plan_peak", (B,), torch.int64), ("verdict", (B,), torch.int32),
                      ("conflict", (2 * B,), torch.int32), ("status", (B,), torch.int32)]
         self.host_in_buf, self.host_in = _packed(in_specs, pin_memory=True)

@@ -21,10 +21,15 @@
 namespace {
 
 // Device buffer layout: inputs, outputs, then the planner's workspace for
-// the largest chunk; every region starts on a kAlign boundary.
+// the largest chunk; every region starts on a kAlign boundary.  The per-trace
+// inputs sit in one region (pertrace, room for trace_ptr, profile_ptr and
+// steps with up to 15 bytes between them) and the per-trace results in
+// another, adjacent in the order peak_lb, plan_peak, verdict, conflict,
+// status, so that each can move in one copy when the host arrays are laid
+// out the same way.
 struct HostPathLayout {
-    size_t trace_ptr, steps, profile_ptr, alloc, free_, size, profile, offsets, peak_lb, plan_peak, verdict,
-        conflict, status, workspace, total;
+    size_t pertrace, alloc, free_, size, profile, offsets, results, peak_lb, plan_peak, verdict, conflict, status,
+        workspace, total;
 };
 
 HostPathLayout host_path_layout(const mp_batch& hb, size_t ws_bytes) {
@@ -38,19 +43,18 @@ HostPathLayout host_path_layout(const mp_batch& hb, size_t ws_bytes) {
         return here;
     };
     using mp::mul_sat;
-    L.trace_ptr = take(mul_sat(B + 1, 8));
-    L.steps = take(mul_sat(B, 4));
-    L.profile_ptr = take(mul_sat(B + 1, 8));
+    L.pertrace = take(mp::add_sat(mul_sat(mul_sat(B + 1, 8), 2), mp::add_sat(mul_sat(B, 4), 32)));
     L.alloc = take(mul_sat(N, 4));
     L.free_ = take(mul_sat(N, 4));
     L.size = take(mul_sat(N, 8));
     L.profile = take(mul_sat(S, 8));
     L.offsets = take(mul_sat(N, 8));
-    L.peak_lb = take(mul_sat(B, 8));
-    L.plan_peak = take(mul_sat(B, 8));
-    L.verdict = take(mul_sat(B, 4));
-    L.conflict = take(mul_sat(B, 8));
-    L.status = take(mul_sat(B, 4));
+    L.results = take(mp::add_sat(mul_sat(B, 16), mul_sat(B, 16)));
+    L.peak_lb = L.results;
+    L.plan_peak = L.peak_lb + (size_t)B * 8;
+    L.verdict = L.plan_peak + (size_t)B * 8;
+    L.conflict = L.verdict + (size_t)B * 4;
+    L.status = L.conflict + (size_t)B * 8;
     L.workspace = take(ws_bytes);
     L.total = at;
     return L;
@@ -249,14 +253,30 @@ __attribute__((visibility("default"))) mp_status mp_plan_and_validate_host(
     auto copy = [&](void* dst, const void* src, size_t bytes, cudaMemcpyKind kind, cudaStream_t s) {
         if (e == cudaSuccess && bytes > 0) e = cudaMemcpyAsync(dst, src, bytes, kind, s);
     };
-    // the per-trace arrays, whole, ahead of the first chunk
-    copy(at<int64_t>(d, L.trace_ptr), hb.trace_ptr, (size_t)(B + 1) * 8, h2d, s_in);
-    copy(at<int32_t>(d, L.steps), hb.steps, (size_t)B * 4, h2d, s_in);
-    copy(at<int64_t>(d, L.profile_ptr), hb.profile_ptr, (size_t)(B + 1) * 8, h2d, s_in);
+    // the per-trace arrays, whole, ahead of the first chunk: one copy when the
+    // host keeps trace_ptr, profile_ptr and steps in this order with fewer
+    // than 16 bytes between them (those bytes are read, never written)
     mp_batch dev = hb;
-    dev.trace_ptr = at<int64_t>(d, L.trace_ptr);
-    dev.steps = at<int32_t>(d, L.steps);
-    dev.profile_ptr = at<int64_t>(d, L.profile_ptr);
+    {
+        const size_t tp = (size_t)(B + 1) * 8, st = (size_t)B * 4;
+        const char* htp = reinterpret_cast<const char*>(hb.trace_ptr);
+        const char* hpp = reinterpret_cast<const char*>(hb.profile_ptr);
+        const char* hst = reinterpret_cast<const char*>(hb.steps);
+        char* dpt = at<char>(d, L.pertrace);
+        if (hpp >= htp + tp && hpp < htp + tp + 16 && hst >= hpp + tp && hst < hpp + tp + 16) {
+            dev.trace_ptr = reinterpret_cast<int64_t*>(dpt);
+            dev.profile_ptr = reinterpret_cast<int64_t*>(dpt + (hpp - htp));
+            dev.steps = reinterpret_cast<int32_t*>(dpt + (hst - htp));
+            copy(dpt, htp, (size_t)(hst - htp) + st, h2d, s_in);
+        } else {
+            dev.trace_ptr = reinterpret_cast<int64_t*>(dpt);
+            dev.profile_ptr = reinterpret_cast<int64_t*>(dpt + tp);
+            dev.steps = reinterpret_cast<int32_t*>(dpt + 2 * tp);
+            copy(dpt, hb.trace_ptr, tp, h2d, s_in);
+            copy(dpt + tp, hb.profile_ptr, tp, h2d, s_in);
+            copy(dpt + 2 * tp, hb.steps, st, h2d, s_in);
+        }
+    }
     dev.alloc_step = at<int32_t>(d, L.alloc);
     dev.free_step = at<int32_t>(d, L.free_);
     dev.size_bytes = at<int64_t>(d, L.size);
@@ -287,12 +307,23 @@ __attribute__((visibility("default"))) mp_status mp_plan_and_validate_host(
         copy(out->offsets + lo, at<int64_t>(d, L.offsets) + lo, (size_t)(hi - lo) * 8, d2h, s_out);
     }
     // the per-trace results, after the last chunk (the copy-out stream has
-    // waited for every chunk's planning by now)
-    copy(out->peak_lb, at<int64_t>(d, L.peak_lb), (size_t)B * 8, d2h, s_out);
-    copy(out->plan_peak, at<int64_t>(d, L.plan_peak), (size_t)B * 8, d2h, s_out);
-    copy(out->verdict, at<int32_t>(d, L.verdict), (size_t)B * 4, d2h, s_out);
-    if (out->conflict != nullptr) copy(out->conflict, at<int32_t>(d, L.conflict), (size_t)B * 8, d2h, s_out);
-    copy(out->trace_status, at<int32_t>(d, L.status), (size_t)B * 4, d2h, s_out);
+    // waited for every chunk's planning by now): one copy when the host
+    // arrays are adjacent in the device block's order, with nothing between
+    // them (a copy back writes every byte it spans)
+    auto bytes_at = [](const void* p) { return reinterpret_cast<const char*>(p); };
+    const bool packed_out = out->conflict != nullptr && bytes_at(out->plan_peak) == bytes_at(out->peak_lb) + B * 8 &&
+                            bytes_at(out->verdict) == bytes_at(out->plan_peak) + B * 8 &&
+                            bytes_at(out->conflict) == bytes_at(out->verdict) + B * 4 &&
+                            bytes_at(out->trace_status) == bytes_at(out->conflict) + B * 8;
+    if (packed_out) {
+        copy(out->peak_lb, at<int64_t>(d, L.results), (size_t)B * 32, d2h, s_out);
+    } else {
+        copy(out->peak_lb, at<int64_t>(d, L.peak_lb), (size_t)B * 8, d2h, s_out);
+        copy(out->plan_peak, at<int64_t>(d, L.plan_peak), (size_t)B * 8, d2h, s_out);
+        copy(out->verdict, at<int32_t>(d, L.verdict), (size_t)B * 4, d2h, s_out);
+        if (out->conflict != nullptr) copy(out->conflict, at<int32_t>(d, L.conflict), (size_t)B * 8, d2h, s_out);
+        copy(out->trace_status, at<int32_t>(d, L.status), (size_t)B * 4, d2h, s_out);
+    }
     return e == cudaSuccess ? MP_OK : MP_ECUDA;
 }
 

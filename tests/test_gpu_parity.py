@@ -635,3 +635,55 @@ def test_breadth_component_tiers(cuda_lib, name, pol):
     assert np.array_equal(st.cpu().numpy(), o_st) and (o_st == 0).all()
     assert np.array_equal(pk.cpu().numpy(), o_pk)
     assert np.array_equal(off.cpu().numpy(), o_off)
+
+
+def test_host_path_against_the_oracle_unpacked(cuda_lib):
+    """mp_plan_and_validate_host through the C ABI with host arrays spaced 64
+    bytes apart and in another order (one copy per array both ways), and with
+    conflict NULL, checked against the oracle directly."""
+    import ctypes
+
+    from paper_2203_00448_gb300 import _lib
+
+    lib = _lib.load()
+    ts = tg.random_small(43, 150, 300, 400, 1 << 28)
+    B, N, S = ts.n_traces, ts.n_tensors, ts.n_steps
+    arrays = [("size_bytes", ts.size_bytes, np.int64), ("steps", ts.steps, np.int32),
+              ("trace_ptr", ts.trace_ptr, np.int64), ("free_step", ts.free_step, np.int32),
+              ("profile_ptr", ts.profile_ptr, np.int64), ("alloc_step", ts.alloc_step, np.int32)]
+    outs = [("status", B, np.int32), ("offsets", N, np.int64), ("verdict", B, np.int32), ("profile", S, np.int64),
+            ("plan_peak", B, np.int64), ("peak_lb", B, np.int64)]
+    total = sum(np.asarray(a).nbytes + 64 for _, a, _ in arrays) + sum(n * np.dtype(d).itemsize + 64 for _, n, d in outs)
+    buf = torch.empty(total + 64, dtype=torch.uint8, pin_memory=True)
+    pos, view = 64, {}
+    for name, a, dt in arrays:
+        a = np.asarray(a, dtype=dt)
+        view[name] = buf[pos:pos + a.nbytes].view(torch.int64 if dt == np.int64 else torch.int32)
+        view[name].numpy()[...] = a
+        pos += a.nbytes + 64
+    for name, n, dt in outs:
+        nbytes = n * np.dtype(dt).itemsize
+        view[name] = buf[pos:pos + nbytes].view(torch.int64 if dt == np.int64 else torch.int32)
+        view[name].fill_(-3)
+        pos += nbytes + 64
+    p = lambda k: view[k].data_ptr()
+    hb = _lib.MpBatch(B, int(ts.max_tensors), int(ts.max_steps), 0, N, S, p("trace_ptr"), p("steps"),
+                      p("profile_ptr"), p("alloc_step"), p("free_step"), p("size_bytes"))
+    res = _lib.MpHostResults(p("profile"), p("peak_lb"), p("offsets"), p("plan_peak"), p("verdict"), None, p("status"))
+    for chunks in (1, 3):
+        need = lib.mp_host_path_bytes(ctypes.byref(hb), chunks)
+        dbuf = torch.empty(need, dtype=torch.uint8, device="cuda")
+        s = torch.cuda.current_stream().cuda_stream
+        st = lib.mp_plan_and_validate_host(ctypes.byref(hb), 0, ctypes.byref(res), chunks, dbuf.data_ptr(),
+                                           dbuf.numel(), s, s, s)
+        assert st == 0
+        torch.cuda.synchronize()
+        o_prof, o_lb, o_st_p = oracle.live_profile(ts)
+        o_off, o_pk, o_st_g = oracle.plan_greedy_by_size(ts, oracle.FIT_FIRST)
+        o_v, _, _ = oracle.validate_plan(ts, o_off)
+        assert (o_st_p == 0).all() and (o_st_g == 0).all()
+        got = {k: view[k].numpy().copy() for k, _, _ in outs}
+        assert np.array_equal(got["status"], o_st_g)
+        for k, want in (("profile", o_prof), ("peak_lb", o_lb), ("offsets", o_off), ("plan_peak", o_pk),
+                        ("verdict", o_v)):
+            assert np.array_equal(got[k], want), (chunks, k)
