@@ -21,9 +21,9 @@
 //     that both precede it and overlap its lifetime (inside an alloc-ordered
 //     run, j < i overlaps i iff f_j > a_i, and j > i iff a_j < f_i); then one
 //     thread per component visits the members in rank order;
-//   - at most kWarpComp tensors: one warp, a tensor per lane; each lane counts
-//     the members that precede it, then the warp places rank 0, 1, ... in
-//     turn with single-instruction warp reductions;
+//   - at most kWarpComp tensors: one warp, a tensor per lane (two per lane
+//     above 32); each lane counts the members that precede it, then the warp
+//     places rank 0, 1, ... in turn with single-instruction warp reductions;
 //   - larger: the whole CTA bitonic-sorts the component into priority order,
 //     then places it tensor by tensor with a CTA-wide gather of the
 //     overlapping placed tensors and a CTA-wide gap search.
@@ -65,7 +65,7 @@ namespace mp {
 namespace {
 
 constexpr int32_t kThreadComp = 8;   // components up to this size: one thread
-constexpr int32_t kWarpComp = 32;    // ... up to this size: one warp (a tensor per lane); else the CTA
+constexpr int32_t kWarpComp = 64;    // ... up to this size: one warp (a tensor or two per lane); else the CTA
 constexpr int kCached = 4;           // tensors per thread kept in registers between the two input passes
 constexpr int32_t kLongLife = 32;    // CTA tier: members living longer than this many steps are listed apart
 constexpr int32_t kPredBuf = 512;    // CTA tier, data in the workspace: predecessors gathered per warp
@@ -327,11 +327,128 @@ __device__ W warp_best_fit(W s, Each&& each) {
     return best;
 }
 
+// Places the component at positions [p0, p0 + c), 32 < c <= 64, with one
+// warp, two tensors per lane (positions lane and lane + 32), as place_warp
+// does with one.  A single component of this size in a CTA holding tiny ones
+// would otherwise go to the CTA tier and outlast every other CTA of its wave.
+template <typename I, typename W>
+__device__ W place_warp2(const ARec<I, W>* AR, W* OFFP, int32_t p0, int32_t c, int32_t policy) {
+    const unsigned full = 0xffffffffu;
+    const int lane = threadIdx.x & 31;
+    bool act[2];
+    W s[2];
+    int32_t a[2], f[2], id[2];
+    int rank[2] = {0, 0};
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+        const int32_t m = lane + 32 * k;
+        act[k] = m < c;
+        s[k] = 0;
+        a[k] = f[k] = 0;
+        id[k] = -1;
+        if (act[k]) {
+            const ARec<I, W> me = AR[p0 + m];
+            s[k] = me.s;
+            a[k] = (int32_t)me.a;
+            f[k] = (int32_t)me.f;
+            id[k] = (int32_t)me.id;
+        }
+    }
+    for (int l = 0; l < 32; ++l) {
+#pragma unroll
+        for (int kk = 0; kk < 2; ++kk) {
+            const W sl = __shfl_sync(full, s[kk], l);
+            const int32_t al = __shfl_sync(full, a[kk], l), il = __shfl_sync(full, id[kk], l);
+            if (l + 32 * kk >= c) continue;
+#pragma unroll
+            for (int k = 0; k < 2; ++k)
+                if (act[k] && !(l == lane && kk == k))
+                    rank[k] += (sl != s[k] ? sl > s[k] : (al != a[k] ? al < a[k] : il < id[k])) ? 1 : 0;
+        }
+    }
+    W off[2] = {0, 0}, end[2] = {0, 0};
+    bool placed[2] = {false, false};
+    for (int r = 0; r < c; ++r) {
+        const unsigned b0 = __ballot_sync(full, act[0] && rank[0] == r);
+        const unsigned b1 = __ballot_sync(full, act[1] && rank[1] == r);
+        const int slot = b0 ? 0 : 1;
+        const int src = __ffs(b0 ? b0 : b1) - 1;
+        const int32_t ai = __shfl_sync(full, slot ? a[1] : a[0], src), fi = __shfl_sync(full, slot ? f[1] : f[0], src);
+        const W si = __shfl_sync(full, slot ? s[1] : s[0], src);
+        bool pred[2];
+#pragma unroll
+        for (int k = 0; k < 2; ++k) pred[k] = placed[k] && a[k] < fi && ai < f[k];  // placed: ranks below r
+        W o = 0;
+        if (policy == MP_FIT_FIRST) {
+            for (;;) {
+                W v = 0;
+#pragma unroll
+                for (int k = 0; k < 2; ++k)
+                    if (pred[k] && off[k] < o + si && o < end[k] && end[k] > v) v = end[k];
+                const W mx = warp_max_w(v);
+                if (mx <= o) break;
+                o = mx;
+            }
+        } else {
+            W t = 0;
+#pragma unroll
+            for (int k = 0; k < 2; ++k)
+                if (pred[k] && end[k] > t) t = end[k];
+            const W top = warp_max_w(t);
+            W cc = 0, best_len = w_none<W>();
+            o = top;
+            while (cc < top) {
+                for (;;) {  // move cc off any predecessor that covers it
+                    W v = 0;
+#pragma unroll
+                    for (int k = 0; k < 2; ++k)
+                        if (pred[k] && off[k] <= cc && cc < end[k] && end[k] > v) v = end[k];
+                    const W mx = warp_max_w(v);
+                    if (mx <= cc) break;
+                    cc = mx;
+                }
+                if (cc >= top) break;
+                W v = w_none<W>();
+#pragma unroll
+                for (int k = 0; k < 2; ++k)
+                    if (pred[k] && off[k] > cc && off[k] < v) v = off[k];
+                const W ns = warp_min_w(v);
+                const W len = ns - cc;
+                if (len >= si && len < best_len) {
+                    best_len = len;
+                    o = cc;
+                }
+                cc = ns;
+            }
+        }
+        if (lane == src) {
+            if (slot == 0) {
+                off[0] = o;
+                end[0] = o + si;
+                placed[0] = true;
+            } else {
+                off[1] = o;
+                end[1] = o + si;
+                placed[1] = true;
+            }
+        }
+    }
+    W mx = 0;
+#pragma unroll
+    for (int k = 0; k < 2; ++k)
+        if (act[k]) {
+            OFFP[p0 + lane + 32 * k] = off[k];
+            mx = end[k] > mx ? end[k] : mx;
+        }
+    return warp_max_w(mx);
+}
+
 // Places the component at positions [p0, p0 + c), c <= 32, with one warp (a
 // tensor per lane); every lane must call it.  Writes OFFP; returns the
 // largest end.
 template <typename I, typename W>
 __device__ W place_warp(const ARec<I, W>* AR, W* OFFP, int32_t p0, int32_t c, int32_t policy) {
+    if (c > 32) return place_warp2(AR, OFFP, p0, c, policy);
     const unsigned full = 0xffffffffu;
     const int lane = threadIdx.x & 31;
     const bool act = lane < c;

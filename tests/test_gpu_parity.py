@@ -687,3 +687,37 @@ def test_host_path_against_the_oracle_unpacked(cuda_lib):
         for k, want in (("profile", o_prof), ("peak_lb", o_lb), ("offsets", o_off), ("plan_peak", o_pk),
                         ("verdict", o_v)):
             assert np.array_equal(got[k], want), (chunks, k)
+
+
+@pytest.mark.parametrize("name,pol", POLICIES)
+def test_two_per_lane_warp_tier(cuda_lib, name, pol):
+    """Components of 33..64 tensors, placed by one warp with two tensors per
+    lane: overlap structures from chains to near-cliques, sizes drawn from few
+    values (ties broken by alloc step and id), in 32-bit traces, traces whose
+    sizes sum past 2^32 (the 64-bit launch), and a batch wide enough in steps
+    to keep its working set in the workspace."""
+    rng = np.random.default_rng(77)
+
+    def comp_trace(c, T, big):
+        a = np.sort(rng.integers(0, T // 2, size=c))
+        f = np.minimum(a + rng.integers(1, T // 2, size=c), T)
+        # keep it one component: every tensor overlaps the next in alloc order
+        for i in range(c - 1):
+            if f[i] <= a[i + 1]:
+                f[i] = a[i + 1] + 1
+        s = rng.choice([64, 128, 192], size=c) * ((1 << 26) if big else 1)
+        return a, f, s
+
+    traces = []
+    for k, c in enumerate([33, 40, 47, 55, 63, 64] * 3):
+        T0 = int(rng.integers(80, 300))
+        a, f, s = comp_trace(c, T0, big=(k % 3 == 2))
+        # a few tiny components after it
+        extra = rng.integers(T0, T0 + 99, size=20)
+        traces.append((T0 + 100, np.concatenate([a, extra]), np.concatenate([f, extra + 1]),
+                       np.concatenate([s, rng.integers(1, 100, size=20) * 8])))
+    ts = tg.from_arrays(traces)
+    assert_parity(ts, gpu_run(ts, name), oracle_run(ts, pol))
+    # the same components with the working set in the workspace (many steps)
+    wide = tg.from_arrays([(T + 40000, a, f, s) for (T, a, f, s) in traces[:6]])
+    assert_parity(wide, gpu_run(wide, name), oracle_run(wide, pol))
