@@ -331,8 +331,9 @@ __device__ W warp_best_fit(W s, Each&& each) {
 // warp, two tensors per lane (positions lane and lane + 32), as place_warp
 // does with one.  A single component of this size in a CTA holding tiny ones
 // would otherwise go to the CTA tier and outlast every other CTA of its wave.
+// Out of line: rarely taken, its code would crowd the hot loop's.
 template <typename I, typename W>
-__device__ W place_warp2(const ARec<I, W>* AR, W* OFFP, int32_t p0, int32_t c, int32_t policy) {
+__device__ __noinline__ W place_warp2(const ARec<I, W>* AR, W* OFFP, int32_t p0, int32_t c, int32_t policy) {
     const unsigned full = 0xffffffffu;
     const int lane = threadIdx.x & 31;
     bool act[2];
