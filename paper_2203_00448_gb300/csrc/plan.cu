@@ -16,11 +16,13 @@
 // is <= alloc(p)).  Each component is then placed by the sequential
 // definition itself:
 //   - one tensor: offset 0;
-//   - at most kThreadComp tensors: one thread.  First, one thread per tensor
-//     finds its priority rank inside its component and the mask of members
-//     that both precede it and overlap its lifetime (inside an alloc-ordered
-//     run, j < i overlaps i iff f_j > a_i, and j > i iff a_j < f_i); then one
-//     thread per component visits the members in rank order;
+//   - at most kThreadComp tensors: one thread.  First, one thread per member
+//     (taken in the size-sorted component list, so that a warp's members
+//     mostly share one component size) finds its priority rank inside its
+//     component and the mask of members that both precede it and overlap its
+//     lifetime (inside an alloc-ordered run, j < i overlaps i iff f_j > a_i,
+//     and j > i iff a_j < f_i); then one thread per component visits the
+//     members in rank order;
 //   - at most kWarpComp tensors: one warp, a tensor per lane (two per lane
 //     above 32); each lane counts the members that precede it, then the warp
 //     places rank 0, 1, ... in turn with single-instruction warp reductions;
@@ -147,7 +149,7 @@ struct PlanLayout {
         bend = main_end > dend ? main_end : dend;
         sb = bend + align16((size_t)T * 4);
         wt = sb + align16((size_t)((n + 31) / 32) * 4);
-        lst = wt + align16((size_t)((n + 31) / 32) * 8);
+        lst = wt + align16((size_t)((n + 31) / 32) * 4);
         rp = lst + align16((size_t)n * 4);  // the thread tier's ranks; later the CTA tier's long-lived ranks
         ord = rp + align16((size_t)n * (cta_tier ? 4 : 2));  // the CTA tier's priority order (int32)
         cnt = ord + (cta_tier ? align16((size_t)n * 4) : 0);  // the CTA tier's predecessor counts (int32)
@@ -1071,20 +1073,10 @@ __device__ W place_heavy(const Comp<I, W>& cp, int32_t k, int32_t policy, int32_
 // ------------------------------------------------------------- components
 
 // Component lookups over the start flags SB (n positions, one bit each).
-// Traces of more than kWordWalk words have per-word tables instead of walks
-// over SB: LW[w] is the last start in words 0..w, and -NW[w] the first start
-// in words w.. (n if none); without tables both are null.
+// Traces of more than kWordWalk words have a per-word table instead of walks
+// over SB: -NW[w] is the first start in words w.. (n if none); without the
+// table NW is null.
 constexpr int32_t kWordWalk = 32;
-
-// Start of the component holding position p.
-__device__ __forceinline__ int32_t comp_start(const uint32_t* SB, const int32_t* LW, int32_t p) {
-    int32_t w = p >> 5;
-    uint32_t m = SB[w] & (0xffffffffu >> (31 - (p & 31)));  // starts at or before p in its word
-    if (m) return (w << 5) + 31 - __clz(m);
-    if (LW) return LW[w - 1];  // position 0 starts a component, so w >= 1 here
-    while (m == 0) m = SB[--w];
-    return (w << 5) + 31 - __clz(m);
-}
 
 // Size of the component starting at position p: distance to the next start.
 __device__ __forceinline__ int32_t comp_size(const uint32_t* SB, const int32_t* NW, int32_t p, int32_t n) {
@@ -1442,6 +1434,8 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
     extern __shared__ __align__(16) unsigned char smem_raw[];
     __shared__ int64_t red[72];
     __shared__ int32_t s_cnt, s_tail, s_bin[kBins], s_base[kBins + 1], s_bad, s_fail, s_big;
+    __shared__ int32_t s_mbase[kBinWarp + 1];  // the thread tier's members, by size class
+    __shared__ uint32_t s_magic[kBinWarp];     // ceil(2^32 / c) of each thread-tier class
     __shared__ unsigned long long s_hi, s_lo, s_max, s_key, s_lbmax;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
     const int32_t policy = out.policy;
@@ -1668,71 +1662,50 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
     }
     __syncthreads();
     const int32_t nwords = (n + 31) >> 5;
-    const int32_t* LW = nullptr;
     const int32_t* NW = nullptr;
-    if (nwords > kWordWalk) {  // per-word tables of the last and the next component start
-        int32_t* lw = WT;
-        int32_t* nw = WT + nwords;
+    if (nwords > kWordWalk) {  // per-word table of the next component start
+        int32_t* nw = WT;
         for (int32_t w = threadIdx.x; w < nwords; w += blockDim.x) {
             const uint32_t m = SB[w];
-            lw[w] = m ? (w << 5) + 31 - __clz(m) : -1;
             nw[w] = m ? -((w << 5) + __ffs(m) - 1) : -n;
         }
         __syncthreads();
-        block_scan_max_i32(lw, nwords, false, reinterpret_cast<int32_t*>(red));
         block_scan_max_i32(nw, nwords, true, reinterpret_cast<int32_t*>(red));
-        LW = lw;
         NW = nw;
     }
 
-    // ---- members, one thread per tensor: a single tensor is placed at 0; a
-    // member of a component of 2..kThreadComp tensors gets its rank and
-    // predecessor mask; component starts are counted by size class
+    // ---- component starts, one thread per tensor: a single tensor is placed
+    // at 0; the starts of larger components are counted by size class
     W mx = 0;
     const unsigned lt_mask = (1u << lane) - 1u;
     for (int32_t q0 = 0; q0 < n; q0 += blockDim.x) {
         const int32_t p = q0 + threadIdx.x;
         int bin = -1;
-        if (p < n) {
-            const int32_t p0 = comp_start(SB, LW, p);
-            const int32_t c = comp_size(SB, NW, p0, n);
+        if (p < n && ((SB[p >> 5] >> (p & 31)) & 1u)) {
+            const int32_t c = comp_size(SB, NW, p, n);
             if (c == 1) {
                 OFFP[p] = 0;
                 mx = max(mx, AR[p].s);
             } else {
-                if (p == p0) {
-                    bin = comp_bin(c);
-                    // the 32-bit launch keeps the CTA tier only with its data in
-                    // shared memory and components up to kDeferComp
-                    if (c > (kSmem ? kDeferComp : kWarpComp)) s_big = 1;
-                }
-                if (c <= kThreadComp) {
-                    const ARec<I, W> me = AR[p];
-                    constexpr bool kPacked = sizeof(W) == 4 && sizeof(I) == 2;
-                    const uint64_t me_key = kPacked ? prio_key(me) : 0;
-                    uint32_t rank = 0, pred = 0;
-                    for (int32_t j = 0; j < c; ++j) {
-                        const int32_t q = p0 + j;
-                        if (q == p) continue;
-                        const ARec<I, W> o = AR[q];
-                        const bool first = kPacked ? precedes_key(o, me_key) : precedes(o, me);
-                        const bool ov = q < p ? (int32_t)o.f > (int32_t)me.a : (int32_t)o.a < (int32_t)me.f;
-                        rank += first ? 1u : 0u;
-                        pred |= (first && ov ? 1u : 0u) << j;
-                    }
-                    RP[p] = (uint16_t)(rank | (pred << 4));
-                }
+                bin = comp_bin(c);
+                // the 32-bit launch keeps the CTA tier only with its data in
+                // shared memory and components up to kDeferComp
+                if (c > (kSmem ? kDeferComp : kWarpComp)) s_big = 1;
             }
         }
         const unsigned grp = __match_any_sync(0xffffffffu, bin);
         if (bin >= 0 && (grp & lt_mask) == 0) atomicAdd(&s_bin[bin], __popc(grp));
     }
     __syncthreads();
-    if (warp == 0) {  // class starts; s_bin becomes each class's cursor
+    if (warp == 0) {  // class starts (s_bin becomes each class's cursor) and the thread tier's member counts
         const int32_t v = lane < kBins ? s_bin[lane] : 0;
         const int32_t incl = warp_incl_scan(v);
         if (lane < kBins) s_base[lane] = s_bin[lane] = incl - v;
         if (lane == kBins - 1) s_base[kBins] = incl;
+        const int32_t mv = lane < kBinWarp ? v * (kThreadComp - lane) : 0;
+        const int32_t mincl = warp_incl_scan(mv);
+        if (lane <= kBinWarp) s_mbase[lane] = mincl - mv;
+        if (lane < kBinWarp) s_magic[lane] = 0xffffffffu / (uint32_t)(kThreadComp - lane) + 1u;
     }
     __syncthreads();
     if constexpr (!kWide) {
@@ -1754,6 +1727,47 @@ __device__ __forceinline__ void plan_trace(const int b, const mp_batch& bt, cons
         if (bin >= 0 && lane == leader) at = atomicAdd(&s_bin[bin], __popc(grp));
         at = __shfl_sync(0xffffffffu, at, leader);
         if (bin >= 0) LST[at + __popc(grp & lt_mask)] = p;
+    }
+    __syncthreads();
+
+    // ---- members of the thread tier's components, one thread per member in
+    // the size-sorted component list (so a warp's members mostly share one
+    // component size): each gets its priority rank and the mask of members
+    // that precede it and overlap its lifetime
+    {
+        int32_t mb[kBinWarp + 1];
+#pragma unroll
+        for (int k = 0; k <= kBinWarp; ++k) mb[k] = s_mbase[k];
+        for (int32_t g = threadIdx.x; g < mb[kBinWarp]; g += blockDim.x) {
+            int bin = 0;
+            int32_t below = 0;  // members of the classes before bin
+#pragma unroll
+            for (int k = 1; k < kBinWarp; ++k) {
+                if (g >= mb[k]) {
+                    bin = k;
+                    below = mb[k];
+                }
+            }
+            const int32_t c = kThreadComp - bin;
+            const uint32_t r = (uint32_t)(g - below);
+            const int32_t k = (int32_t)__umulhi(r, s_magic[bin]);  // r / c (r < 2^28)
+            const int32_t p0 = LST[s_base[bin] + k];
+            const int32_t p = p0 + ((int32_t)r - k * c);
+            const ARec<I, W> me = AR[p];
+            constexpr bool kPacked = sizeof(W) == 4 && sizeof(I) == 2;
+            const uint64_t me_key = kPacked ? prio_key(me) : 0;
+            uint32_t rank = 0, pred = 0;
+            for (int32_t j = 0; j < c; ++j) {
+                const int32_t q = p0 + j;
+                if (q == p) continue;
+                const ARec<I, W> o = AR[q];
+                const bool first = kPacked ? precedes_key(o, me_key) : precedes(o, me);
+                const bool ov = q < p ? (int32_t)o.f > (int32_t)me.a : (int32_t)o.a < (int32_t)me.f;
+                rank += first ? 1u : 0u;
+                pred |= (first && ov ? 1u : 0u) << j;
+            }
+            RP[p] = (uint16_t)(rank | (pred << 4));
+        }
     }
     __syncthreads();
 
