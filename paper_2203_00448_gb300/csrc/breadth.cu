@@ -483,6 +483,8 @@ k_breadth_comp(mp_batch bt, int32_t policy, int64_t* __restrict__ offsets, int64
     extern __shared__ __align__(16) unsigned char smem_raw[];
     __shared__ int64_t red[72];
     __shared__ int32_t s_bad, s_defer, s_nt, s_nw, s_nb, s_cnt, s_bin[kBThreadComp - 1], s_base[kBThreadComp];
+    __shared__ int32_t s_mbase[kBThreadComp];    // the thread tier's members, by size class
+    __shared__ uint32_t s_magic[kBThreadComp - 1];  // ceil(2^32 / c) of each size class
     __shared__ int32_t s_big[kBBigComps];
     __shared__ unsigned long long s_hi, s_lo;
     const int b = blockIdx.x;
@@ -577,8 +579,7 @@ k_breadth_comp(mp_batch bt, int32_t policy, int64_t* __restrict__ offsets, int64
         }
     }
     __syncthreads();
-    // every member finds its component; a single tensor sits at 0; a member
-    // of a thread-tier component gets its rank and predecessor mask; the
+    // every component start finds its size: a single tensor sits at 0; the
     // components are counted by tier and size
     auto size_from = [&](int32_t p0) {  // distance from a start to the next one
         int32_t w = p0 >> 5;
@@ -587,14 +588,68 @@ k_breadth_comp(mp_batch bt, int32_t policy, int64_t* __restrict__ offsets, int64
         return (m ? (w << 5) + __ffs(m) - 1 : n) - p0;
     };
     for (int32_t p = tid; p < n; p += nthr) {
-        int32_t w = p >> 5;
-        uint32_t m = SB[w] & (0xffffffffu >> (31 - (p & 31)));  // starts at or before p
-        while (m == 0) m = SB[--w];                              // position 0 is a start
-        const int32_t p0 = (w << 5) + 31 - __clz(m);
-        const int32_t c = size_from(p0);
+        if (!((SB[p >> 5] >> (p & 31)) & 1u)) continue;
+        const int32_t c = size_from(p);
         if (c == 1) {
             OFF[p] = 0;
         } else if (c <= kBThreadComp) {
+            atomicAdd(&s_bin[kBThreadComp - c], 1);
+        } else if (c <= kBWarpComp) {
+            LST[n - 1 - atomicAdd(&s_nw, 1)] = p * 64 + c;
+        } else {  // the CTA tier, while its scratch holds the component
+            const int32_t at = atomicAdd(&s_nb, 1);
+            if (at < kBBigComps && big_fits(c, T)) s_big[at] = p;
+            else s_defer = 1;
+        }
+    }
+    __syncthreads();
+    if (s_defer) {  // too many large components, or one too large: the per-tensor kernel places this trace
+        if (tid == 0) status[b] = kBDeferred;
+        return;
+    }
+    if (tid == 0) {  // thread-tier components in descending size: bin starts, then cursors; member counts
+        int32_t at = 0, mat = 0;
+        for (int32_t k = 0; k < kBThreadComp - 1; ++k) {
+            s_base[k] = at;
+            s_mbase[k] = mat;
+            s_magic[k] = 0xffffffffu / (uint32_t)(kBThreadComp - k) + 1u;
+            at += s_bin[k];
+            mat += s_bin[k] * (kBThreadComp - k);
+            s_bin[k] = s_base[k];
+        }
+        s_nt = at;
+        s_mbase[kBThreadComp - 1] = mat;
+    }
+    __syncthreads();
+    for (int32_t p = tid; p < n; p += nthr) {
+        if (!((SB[p >> 5] >> (p & 31)) & 1u)) continue;
+        const int32_t c = size_from(p);
+        if (c >= 2 && c <= kBThreadComp) LST[atomicAdd(&s_bin[kBThreadComp - c], 1)] = p * 64 + c;
+    }
+    __syncthreads();
+    // members of the thread tier's components, one thread per member in the
+    // size-sorted component list (so a warp's members mostly share one
+    // component size): each gets its rank in the breadth order and the mask
+    // of the earlier-ranked members that overlap its lifetime
+    {
+        int32_t mb[kBThreadComp];
+#pragma unroll
+        for (int k = 0; k < kBThreadComp; ++k) mb[k] = s_mbase[k];
+        for (int32_t g = tid; g < mb[kBThreadComp - 1]; g += nthr) {
+            int bin = 0;
+            int32_t below = 0;  // members of the classes before bin
+#pragma unroll
+            for (int k = 1; k < kBThreadComp - 1; ++k) {
+                if (g >= mb[k]) {
+                    bin = k;
+                    below = mb[k];
+                }
+            }
+            const int32_t c = kBThreadComp - bin;
+            const uint32_t r = (uint32_t)(g - below);
+            const int32_t k = (int32_t)__umulhi(r, s_magic[bin]);  // r / c (r < 2^28)
+            const int32_t p0 = LST[s_base[bin] + k] >> 6;
+            const int32_t p = p0 + ((int32_t)r - k * c);
             const BRec me = R[p];
             uint32_t rank = 0, mask = 0;
             for (int32_t j = 0; j < c; ++j) {
@@ -607,34 +662,7 @@ k_breadth_comp(mp_batch bt, int32_t policy, int64_t* __restrict__ offsets, int64
             }
             RK[p] = (int32_t)(mask << 8 | rank);
             BYR[p0 + rank] = (uint8_t)(p - p0);
-            if (p == p0) atomicAdd(&s_bin[kBThreadComp - c], 1);
-        } else if (c <= kBWarpComp) {
-            if (p == p0) LST[n - 1 - atomicAdd(&s_nw, 1)] = p0 * 64 + c;
-        } else if (p == p0) {  // the CTA tier, while its scratch holds the component
-            const int32_t at = atomicAdd(&s_nb, 1);
-            if (at < kBBigComps && big_fits(c, T)) s_big[at] = p0;
-            else s_defer = 1;
         }
-    }
-    __syncthreads();
-    if (s_defer) {  // too many large components, or one too large: the per-tensor kernel places this trace
-        if (tid == 0) status[b] = kBDeferred;
-        return;
-    }
-    if (tid == 0) {  // thread-tier components in descending size: bin starts, then cursors
-        int32_t at = 0;
-        for (int32_t k = 0; k < kBThreadComp - 1; ++k) {
-            s_base[k] = at;
-            at += s_bin[k];
-            s_bin[k] = s_base[k];
-        }
-        s_nt = at;
-    }
-    __syncthreads();
-    for (int32_t p = tid; p < n; p += nthr) {
-        if (!((SB[p >> 5] >> (p & 31)) & 1u)) continue;
-        const int32_t c = size_from(p);
-        if (c >= 2 && c <= kBThreadComp) LST[atomicAdd(&s_bin[kBThreadComp - c], 1)] = p * 64 + c;
     }
     __syncthreads();
     for (int32_t i = warp; i < s_nw; i += nwarps) {
