@@ -145,27 +145,22 @@ __device__ __forceinline__ void check_pairs_wide(const longlong2* __restrict__ r
     }
 }
 
-// One CTA per trace.  The first kValCached * blockDim tensors are loaded into
-// registers before anything else (16-byte loads when the trace's slices are
-// aligned) and kept there for the scatter, so a trace's inputs are read from
-// memory once; larger traces read the rest twice.  Traces whose ends all lie
+// One CTA per trace.  A trace of at most kValCached * blockDim tensors is
+// loaded into registers before anything else (16-byte loads when its slices
+// are aligned) and kept there for the scatter, so its inputs are read from
+// memory once; a larger trace is read twice, by plain loops.  The two cases
+// are separate code paths (kCached), so that no cached value is live across
+// a loop that reads memory: inlined together, those loops made the kernel
+// spill registers even for traces that never ran them.  Traces whose ends all lie
 // below 2^32 (the flag reduction tells) take 8-byte records and 32-bit
 // compares; the exact size sum is only formed when some size reaches 2^32
 // (below that, n < 2^31 sizes cannot sum past INT64_MAX).
-template <bool kSmem>
-__global__ void __launch_bounds__(kValidateThreads, kSmem ? 9 : 1)
-k_validate(mp_batch bt, const int64_t* __restrict__ offsets, int32_t* __restrict__ verdict,
-           int32_t* __restrict__ conflict, int32_t* __restrict__ status, unsigned char* __restrict__ ws,
-           size_t ws_stride) {
-    extern __shared__ __align__(16) unsigned char smem_raw[];
-    __shared__ int32_t red[40];
-    __shared__ ValidateShared sh;
-    const int b = blockIdx.x;
-    const TraceView tv = load_trace(bt, b, false);
-    if (tv.st != MP_OK) {
-        if (threadIdx.x == 0) status[b] = tv.st;
-        return;
-    }
+template <bool kSmem, bool kCached>
+__device__ __forceinline__ void validate_trace(const mp_batch& bt, const TraceView& tv, int b,
+                                               const int64_t* __restrict__ offsets, int32_t* __restrict__ verdict,
+                                               int32_t* __restrict__ conflict, int32_t* __restrict__ status,
+                                               unsigned char* __restrict__ ws, size_t ws_stride,
+                                               unsigned char* smem_raw, int32_t* red, ValidateShared& sh) {
     const int32_t n = tv.n, T = tv.T;
     const int32_t tid = (int32_t)threadIdx.x, nthr = (int32_t)blockDim.x;
     const int32_t* __restrict__ Ag = bt.alloc_step + tv.lo;
@@ -175,9 +170,11 @@ k_validate(mp_batch bt, const int64_t* __restrict__ offsets, int32_t* __restrict
     const bool vec = ((reinterpret_cast<uintptr_t>(Ag) | reinterpret_cast<uintptr_t>(Fg) |
                        reinterpret_cast<uintptr_t>(Sg) | reinterpret_cast<uintptr_t>(Og)) & 15) == 0;
     auto cidx = [&](int j) -> int32_t { return vec ? 4 * tid + j : tid + j * nthr; };
-    int32_t ca[kValCached], cf[kValCached];
-    int64_t cs[kValCached], co[kValCached];
-    if (vec && 4 * tid + 3 < n) {
+    int32_t ca[kValCached] = {}, cf[kValCached] = {};
+    int64_t cs[kValCached] = {}, co[kValCached] = {};
+    if (!kCached) {
+        // nothing held: every tensor is read by the loops below
+    } else if (vec && 4 * tid + 3 < n) {
         const int4 a = __ldg(reinterpret_cast<const int4*>(Ag) + tid);
         const int4 f = __ldg(reinterpret_cast<const int4*>(Fg) + tid);
         const longlong2 s01 = __ldg(reinterpret_cast<const longlong2*>(Sg) + 2 * tid);
@@ -236,14 +233,16 @@ k_validate(mp_batch bt, const int64_t* __restrict__ offsets, int32_t* __restrict
         if (ok) atomicAdd(BEND + a, 1);
         return e;
     };
-    uint32_t co32[kValCached], ce32[kValCached];
+    uint32_t co32[kValCached] = {}, ce32[kValCached] = {};
+    if constexpr (kCached) {
 #pragma unroll
-    for (int j = 0; j < kValCached; ++j) {
-        co32[j] = (uint32_t)co[j];
-        ce32[j] = cidx(j) < n ? (uint32_t)take(ca[j], cf[j], cs[j], co[j]) : 0u;
+        for (int j = 0; j < kValCached; ++j) {
+            co32[j] = (uint32_t)co[j];
+            ce32[j] = cidx(j) < n ? (uint32_t)take(ca[j], cf[j], cs[j], co[j]) : 0u;
+        }
+    } else {
+        for (int32_t k = tid; k < n; k += nthr) take(__ldg(Ag + k), __ldg(Fg + k), __ldg(Sg + k), __ldg(Og + k));
     }
-    const int32_t nc = min(n, kValCached * nthr);
-    for (int32_t k = nc + tid; k < n; k += nthr) take(__ldg(Ag + k), __ldg(Fg + k), __ldg(Sg + k), __ldg(Og + k));
     int flags = (bad ? kFlagInvalid : 0) | ((or_e >> 63) ? kFlagEndOvf : 0) | ((or_e >> 32) ? kFlagWide : 0) |
                 ((or_s >> 32) ? kFlagBigSize : 0);
     flags = (int)__reduce_or_sync(0xffffffffu, (unsigned)flags);
@@ -282,14 +281,17 @@ k_validate(mp_batch bt, const int64_t* __restrict__ offsets, int32_t* __restrict
             REC32[pos] = make_uint4(o32, e32, (uint32_t)f, (uint32_t)k);
         }
     };
+    if constexpr (kCached) {
 #pragma unroll
-    for (int j = 0; j < kValCached; ++j) {
-        const int32_t k = cidx(j);
-        if (k < n) scatter(k, ca[j], cf[j], co32[j], ce32[j]);
-    }
-    for (int32_t k = nc + tid; k < n; k += nthr) {
-        const uint32_t o32 = wide ? 0u : (uint32_t)__ldg(Og + k);
-        scatter(k, __ldg(Ag + k), __ldg(Fg + k), o32, wide ? 0u : o32 + (uint32_t)__ldg(Sg + k));
+        for (int j = 0; j < kValCached; ++j) {
+            const int32_t k = cidx(j);
+            if (k < n) scatter(k, ca[j], cf[j], co32[j], ce32[j]);
+        }
+    } else {
+        for (int32_t k = tid; k < n; k += nthr) {
+            const uint32_t o32 = wide ? 0u : (uint32_t)__ldg(Og + k);
+            scatter(k, __ldg(Ag + k), __ldg(Fg + k), o32, wide ? 0u : o32 + (uint32_t)__ldg(Sg + k));
+        }
     }
     __syncthreads();
 
@@ -308,6 +310,27 @@ k_validate(mp_batch bt, const int64_t* __restrict__ offsets, int32_t* __restrict
         }
         status[b] = MP_OK;
     }
+}
+
+template <bool kSmem>
+__global__ void __launch_bounds__(kValidateThreads, kSmem ? 9 : 1)
+k_validate(mp_batch bt, const int64_t* __restrict__ offsets, int32_t* __restrict__ verdict,
+           int32_t* __restrict__ conflict, int32_t* __restrict__ status, unsigned char* __restrict__ ws,
+           size_t ws_stride) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    __shared__ int32_t red[40];
+    __shared__ ValidateShared sh;
+    const int b = blockIdx.x;
+    const TraceView tv = load_trace(bt, b, false);
+    if (tv.st != MP_OK) {
+        if (threadIdx.x == 0) status[b] = tv.st;
+        return;
+    }
+    if (tv.n <= kValCached * (int32_t)blockDim.x)
+        validate_trace<kSmem, true>(bt, tv, b, offsets, verdict, conflict, status, ws, ws_stride, smem_raw, red, sh);
+    else
+        validate_trace<kSmem, false>(bt, tv, b, offsets, verdict, conflict, status, ws, ws_stride, smem_raw, red,
+                                     sh);
 }
 
 __global__ void __launch_bounds__(kPeakThreads)
